@@ -1,0 +1,353 @@
+"""Pins of the fp64 oracle against facts fixed by the paper and by mathematics.
+
+Each ``pin_*`` takes the oracle module (so the same checks can be run on a
+copy of it with a planted mistake) and raises AssertionError on a violation.
+None of them re-types the oracle's formula: they use closed forms, invariants,
+hand-worked values (``tests/golden``), independent formulations and library
+routines for special cases.
+"""
+
+from __future__ import annotations
+
+import itertools
+import json
+import math
+import os
+from fractions import Fraction
+
+import numpy as np
+from scipy.ndimage import maximum_filter1d
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+def _golden(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return json.load(f)
+
+
+def _bf16_bits(x):
+    """float -> bf16 bits, for values that are exactly representable."""
+    f = np.asarray(x, dtype=np.float32)
+    bits = f.view(np.uint32)
+    assert np.all((bits & 0xFFFF) == 0), "value not exact in bf16"
+    return (bits >> 16).astype(np.uint16)
+
+
+def _harmonic(m):
+    return sum(Fraction(1, j) for j in range(1, m + 1))
+
+
+# ---------------------------------------------------------------- softmax ---
+
+def pin_rows_sum_to_one(O, rng):
+    """Every causal softmax row sums to 1 and puts no mass after its position."""
+    n, d = 57, 16
+    q = rng.standard_normal((9, d)) * 2
+    k = rng.standard_normal((n, d)) * 2
+    pos = np.array([0, 3, 10, 20, 33, 40, 50, 55, 56])
+    P = O.attention_probs(q, k, pos, 1 / math.sqrt(d))
+    assert np.allclose(P.sum(axis=1), 1.0, rtol=0, atol=1e-12)
+    for r, p in enumerate(pos):
+        assert np.all(P[r, p + 1:] == 0)
+        assert np.all(P[r, :p + 1] > 0)
+
+
+def pin_snapkv_total(O, rng):
+    """SnapKV pre-pool mass of a unit totals W_eff * G (every window row is a
+    probability distribution), for W < n and W > n."""
+    d, G = 16, 3
+    for n, W in ((40, 8), (5, 8), (64, 64)):
+        qw = rng.standard_normal((G, W, d))
+        k = rng.standard_normal((n, d))
+        s = O.snapkv_prepool(qw, k, W, 1 / math.sqrt(d))
+        assert s.shape == (n,)
+        assert abs(s.sum() - min(W, n) * G) < 1e-10
+
+
+def pin_h2o_total(O, rng):
+    """H2O mass of a unit totals n * G (one distribution per causal query)."""
+    d, G, n = 16, 2, 37
+    q = rng.standard_normal((G, n, d))
+    k = rng.standard_normal((n, d))
+    s = O.h2o_score(q, k, 1 / math.sqrt(d))
+    assert abs(s.sum() - n * G) < 1e-10
+
+
+def pin_uniform_closed_forms(O, rng):
+    """Identical keys give uniform attention over each causal prefix, so
+    SnapKV s(t) = G * sum over window positions p >= t of 1/(p+1) and
+    H2O s(t) = G * (H_n - H_t), H the harmonic numbers."""
+    d, G, n, W = 8, 2, 23, 6
+    k = np.tile(rng.standard_normal(d), (n, 1))
+    qw = rng.standard_normal((G, W, d))
+    s = O.snapkv_prepool(qw, k, W, 1 / math.sqrt(d))
+    window = range(n - W, n)
+    for t in range(n):
+        exact = G * sum(Fraction(1, p + 1) for p in window if p >= t)
+        assert abs(s[t] - float(exact)) < 1e-12, (t, s[t], float(exact))
+    q = rng.standard_normal((G, n, d))
+    h = O.h2o_score(q, k, 1 / math.sqrt(d))
+    Hn = _harmonic(n)
+    for t in range(n):
+        exact = G * (Hn - _harmonic(t))
+        assert abs(h[t] - float(exact)) < 1e-12, (t, h[t], float(exact))
+
+
+def _two_level_prob(z, n_hot, n_cold):
+    """Softmax of n_hot logits z and n_cold logits 0: (p_hot, p_cold)."""
+    den = n_hot * math.exp(z) + n_cold
+    return math.exp(z) / den, 1.0 / den
+
+
+def pin_two_level_scale(O, rng):
+    """Keys c*e0 on a set A and 0 elsewhere, queries x*e0: the logit on A is
+    z = x*c/sqrt(d), which fixes the softmax scale 1/sqrt(d)."""
+    d, n, W, G = 64, 30, 5, 1
+    x, c = 2.0, 2.0
+    A = {1, 4, 9, 27, 28}
+    k = np.zeros((n, d))
+    for t in A:
+        k[t, 0] = c
+    qw = np.zeros((G, W, d))
+    qw[:, :, 0] = x
+    z = x * c / math.sqrt(d)
+    s = O.snapkv_prepool(qw, k, W, 1 / math.sqrt(d))
+    expect = np.zeros(n)
+    for p in range(n - W, n):
+        n_hot = sum(1 for t in A if t <= p)
+        ph, pc = _two_level_prob(z, n_hot, p + 1 - n_hot)
+        for t in range(p + 1):
+            expect[t] += ph if t in A else pc
+    assert np.allclose(s, expect, rtol=1e-12, atol=0)
+
+
+def pin_window_covering_is_h2o(O, rng):
+    """With W >= n every query is in the window, so SnapKV equals H2O."""
+    d, G, n = 16, 2, 19
+    q = rng.standard_normal((G, n, d))
+    k = rng.standard_normal((n, d))
+    qw = np.zeros((G, 24, d))
+    qw[:, :n, :] = q
+    a = O.snapkv_prepool(qw, k, 24, 0.3)
+    b = O.h2o_score(q, k, 0.3)
+    assert np.allclose(a, b, rtol=1e-12, atol=1e-14)
+
+
+def pin_gqa_grouping(O, rng):
+    """Query heads h*G .. h*G+G-1 share KV head h (grouped-query attention).
+    KV head 0 has identical keys (uniform closed form whatever the queries);
+    KV head 1 has one hot key at t=0 and its group's queries point at it."""
+    L, b, Hq, Hkv, d, n, W = 1, 1, 4, 2, 8, 16, 4
+    G = Hq // Hkv
+    k = np.zeros((L, b, Hkv, n, d))
+    k[0, 0, 0, :, :] = 1.0
+    k[0, 0, 1, 0, 0] = 4.0
+    qw = np.zeros((L, b, Hq, W, d))
+    qw[0, 0, 0:2] = rng.choice([-1.0, 1.0, 2.0], size=(2, W, d))
+    qw[0, 0, 2:4, :, 0] = 2.0
+    batch = O.Batch(L, b, Hq, Hkv, d, n)
+    res = O.snapkv_batch(batch, _bf16_bits(qw), _bf16_bits(k), W, 1, scale=1 / math.sqrt(d))
+    s0 = res[0][0]
+    for t in range(n):
+        exact = G * sum(Fraction(1, p + 1) for p in range(n - W, n) if p >= t)
+        assert abs(s0[t] - float(exact)) < 1e-12
+    s1 = res[1][0]
+    z = 2.0 * 4.0 / math.sqrt(d)
+    expect = np.zeros(n)
+    for p in range(n - W, n):
+        ph, pc = _two_level_prob(z, 1, p)
+        expect[0] += G * ph
+        expect[1:p + 1] += G * pc
+    assert np.allclose(s1, expect, rtol=1e-12, atol=0)
+
+
+# ---------------------------------------------------------------- pooling ---
+
+def pin_maxpool(O, rng):
+    """Hand-worked pools, the k=1 identity, s~ >= s, and scipy's
+    maximum_filter1d with -inf padding as an independent routine."""
+    g = _golden("maxpool_worked_examples.json")
+    s = np.array(g["s"], dtype=np.float64)
+    for case in g["cases"]:
+        assert np.array_equal(O.maxpool1d(s, case["k"]), np.array(case["out"], dtype=np.float64))
+    x = rng.random(101)
+    assert np.array_equal(O.maxpool1d(x, 1), x)
+    for k in (3, 5, 7, 11, 15):
+        y = O.maxpool1d(x, k)
+        assert np.all(y >= x)
+        ref = maximum_filter1d(x, size=k, mode="constant", cval=-np.inf)
+        assert np.array_equal(y, ref)
+    short = rng.random(2)
+    assert np.array_equal(O.maxpool1d(short, 7), np.full(2, short.max()))
+
+
+# ---------------------------------------------------------------- budget ----
+
+def pin_kept_count(O, rng):
+    g = _golden("quota_worked_examples.json")["kept_count"]
+    for n, B, k in g["cases"]:
+        assert O.kept_count(n, B) == k, (n, B, O.kept_count(n, B), k)
+    for n in (1, 2, 3, 1000, 32768, 100003):
+        for B in (0.05, 0.1, 0.2, 0.3, 0.5, 0.75, 1.0):
+            k = O.kept_count(n, B)
+            exact = Fraction(round(B * 1e6), 10**6) * n
+            assert k == math.ceil(exact), (n, B, k)
+
+
+def pin_quota_golden(O, rng):
+    g = _golden("quota_worked_examples.json")
+    for ex in g["examples"]:
+        q = O.role_quotas(ex["counts"], ex["alpha"], ex["budget"], ex["n"])
+        assert q == ex["quotas"], (ex["name"], q, ex["quotas"])
+        assert sum(q) == ex["kept"]
+
+
+def _water_level(counts, weights, K):
+    """Independent formulation: the ideal (real-valued) split is
+    x_r = min(n_r, w_r * lam) with lam chosen so that sum x_r = K; lam is
+    found by walking the breakpoints n_r / w_r in increasing order."""
+    live = [r for r in range(len(counts)) if weights[r] > 0 and counts[r] > 0]
+    if K == 0 or not live:
+        return {r: Fraction(0) for r in live}
+    order = sorted(live, key=lambda r: Fraction(counts[r], weights[r]))
+    fixed_sum, free_w = 0, sum(weights[r] for r in live)
+    for i, r in enumerate(order):
+        lam = Fraction(K - fixed_sum, free_w)
+        if weights[r] * lam <= counts[r]:
+            break
+        fixed_sum += counts[r]
+        free_w -= weights[r]
+    else:
+        return {r: Fraction(counts[r]) for r in live}
+    return {r: min(Fraction(counts[r]), weights[r] * lam) for r in live}
+
+
+def pin_quota_waterlevel(O, rng):
+    """Quotas sum to K = min(ceil(B n), eligible), never exceed a bucket,
+    equal the bucket size where the ideal split saturates it, and otherwise
+    lie within one of the exact rational ideal split."""
+    for _ in range(400):
+        R = int(rng.integers(1, 9))
+        counts = [int(x) for x in rng.integers(0, 60, size=R)]
+        if rng.random() < 0.3:
+            counts[int(rng.integers(R))] = 0
+        n = sum(counts)
+        if n == 0:
+            continue
+        alpha = [float(np.float32(x)) for x in rng.choice([0.0, 0.02, 0.05, 0.2, 0.25, 0.7, 0.33], size=R)]
+        B = float(rng.choice([0.05, 0.1, 0.2, 0.3, 0.5, 0.9, 1.0]))
+        q = O.role_quotas(counts, alpha, B, n)
+        w = [round(a * 1e6) for a in alpha]
+        elig = sum(c for c, a in zip(counts, w) if a > 0)
+        K = min(math.ceil(Fraction(round(B * 1e6), 10**6) * n), elig)
+        assert sum(q) == K, (counts, alpha, B, q, K)
+        ideal = _water_level(counts, w, K)
+        for r in range(R):
+            assert 0 <= q[r] <= counts[r]
+            if r not in ideal:
+                assert q[r] == 0
+                continue
+            x = ideal[r]
+            assert math.floor(x) <= q[r] <= math.ceil(x), (counts, alpha, B, q, r, x)
+
+
+def pin_key_ban(O, rng):
+    """alpha_KEY = 0 keeps no KEY token (the role the method is built to zero,
+    Section 4.1 'Hyperparameters'), whatever the scores."""
+    b, n, Hkv = 2, 300, 2
+    batch = O.Batch(1, b, Hkv * 2, Hkv, 8, n)
+    roles = rng.integers(0, 4, size=(b, n)).astype(np.uint8)
+    scores = {}
+    for u in range(batch.n_units):
+        _, s, _ = batch.unit(u)
+        sc = rng.random(n)
+        sc[roles[s] == 1] += 100.0    # KEY tokens score highest
+        scores[u] = sc
+    for B in (0.05, 0.2, 0.5, 0.9):
+        res = O.select_batch(batch, scores, roles, 4, [0.25, 0.5, 0.70, 0.05], 1, 0.0, B)
+        for u, (idx, per_role) in res.items():
+            _, s, _ = batch.unit(u)
+            kept = idx[idx >= 0]
+            assert per_role[1] == 0
+            assert np.all(roles[s][kept] != 1)
+            elig = int((roles[s] != 1).sum())
+            assert kept.size == min(math.ceil(Fraction(round(B * 1e6), 10**6) * n), elig)
+            assert np.all(np.diff(kept) > 0)
+
+
+def pin_global_is_full_sort(O, rng):
+    """GLOBAL policy with no ban is plain top-K by score with ties to the
+    lower index: numpy's stable argsort of -score, first K, sorted."""
+    n = 500
+    for trial in range(6):
+        sc = rng.integers(0, 40, size=n).astype(np.float64)   # many ties
+        roles = rng.integers(0, 4, size=n)
+        for B in (0.05, 0.2, 0.5):
+            K = O.kept_count(n, B)
+            q = O.role_quotas([int((roles == r).sum()) for r in range(4)], [1, 1, 1, 1], B, n,
+                              policy=O.POLICY_GLOBAL)
+            bk = O.bucket_of_tokens(roles, O.POLICY_GLOBAL, 0)
+            idx = O.select_unit(sc, bk, q)
+            ref = np.sort(np.argsort(-sc, kind="stable")[:K])
+            assert np.array_equal(idx, ref)
+
+
+def pin_bruteforce_select(O, rng):
+    """For tiny units, each bucket's kept set is the subset of its size that
+    maximises the score sum, and among those the smallest index tuple
+    (exhaustive enumeration, integer scores so sums are exact)."""
+    for trial in range(25):
+        n = int(rng.integers(6, 15))
+        roles = rng.integers(0, 3, size=n)
+        sc = rng.integers(0, 5, size=n).astype(np.float64)
+        counts = [int((roles == r).sum()) for r in range(3)]
+        B = float(rng.choice([0.2, 0.3, 0.5, 0.7]))
+        q = O.role_quotas(counts, [0.5, 0.3, 0.2], B, n)
+        idx = O.select_unit(sc, roles, q)
+        for r in range(3):
+            members = [int(t) for t in np.nonzero(roles == r)[0]]
+            best = None
+            for sub in itertools.combinations(members, q[r]):
+                key = (-sum(sc[list(sub)]), sub)
+                best = key if best is None or key < best else best
+            chosen = tuple(int(t) for t in idx if roles[t] == r)
+            assert chosen == best[1], (trial, r, chosen, best)
+
+
+def pin_compact(O, rng):
+    """Compaction is numpy's take on the token axis; -1 gives a zero row."""
+    rows = rng.integers(0, 2**16, size=(50, 8)).astype(np.uint16)
+    idx = np.array([0, 3, 4, 17, 49, -1, -1])
+    out = O.compact_unit(rows, idx)
+    assert np.array_equal(out[:5], np.take(rows, idx[:5], axis=0))
+    assert np.all(out[5:] == 0)
+
+
+def pin_varlen_matches_dense(O, rng):
+    """The packed (varlen) layout gives the same per-unit scores as the dense
+    layout when every sequence has the same length."""
+    L, b, Hq, Hkv, d, n, W = 2, 3, 4, 2, 8, 12, 4
+    kd = rng.integers(0x3c00, 0x4000, size=(L, b, Hkv, n, d)).astype(np.uint16)
+    qd = rng.integers(0x3c00, 0x4000, size=(L, b, Hq, n, d)).astype(np.uint16)
+    qw = rng.integers(0x3c00, 0x4000, size=(L, b, Hq, W, d)).astype(np.uint16)
+    kv = np.ascontiguousarray(np.transpose(kd, (0, 1, 3, 2, 4)).reshape(L, b * n, Hkv, d))
+    qv = np.ascontiguousarray(np.transpose(qd, (0, 1, 3, 2, 4)).reshape(L, b * n, Hq, d))
+    dense = O.Batch(L, b, Hq, Hkv, d, n)
+    var = O.Batch(L, b, Hq, Hkv, d, n, seqlens=[n] * b)
+    a = O.snapkv_batch(dense, qw, kd, W, 3)
+    c = O.snapkv_batch(var, qw, kv, W, 3)
+    for u in a:
+        assert np.array_equal(a[u][1], c[u][1])
+    a = O.h2o_batch(dense, qd, kd)
+    c = O.h2o_batch(var, qv, kv)
+    for u in a:
+        assert np.allclose(a[u], c[u], rtol=1e-14, atol=0)
+
+
+ALL_PINS = [
+    pin_rows_sum_to_one, pin_snapkv_total, pin_h2o_total, pin_uniform_closed_forms,
+    pin_two_level_scale, pin_window_covering_is_h2o, pin_gqa_grouping, pin_maxpool,
+    pin_kept_count, pin_quota_golden, pin_quota_waterlevel, pin_key_ban,
+    pin_global_is_full_sort, pin_bruteforce_select, pin_compact, pin_varlen_matches_dense,
+]

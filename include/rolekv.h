@@ -1,0 +1,221 @@
+/*
+ * rolekv.h -- C ABI of librolekv: the data-parallel hot path of
+ * role-conditional KV-cache eviction (arXiv 2607.13205, "Adaptive Filtering of
+ * the KV Cache").
+ *
+ * Pipeline (Algorithm 1, per layer and KV head):
+ *   snapkv_score      windowed attention mass of the last W queries, GQA heads
+ *                     summed, then the 1-D max-pool along the KV axis;
+ *   h2o_score         the H2O accumulated mass s(t) = sum_q p_t(q) it is
+ *                     compared against (Section 2);
+ *   role_alloc_select per-role-bucket top-k under the budget B, split by the
+ *                     role weights alpha with the single tuned knob alpha_KEY
+ *                     (Section 4.1);
+ *   kv_compact        gather of the kept K/V rows into a dense cache (the
+ *                     compacting implementation of Section 6).
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * Units.  One unit is one (layer l, sequence s, KV head h); units are numbered
+ *   u = (l * b + s) * Hkv + h.  Query head hq belongs to KV head hq / G with
+ *   G = Hq / Hkv (grouped-query attention, consecutive heads share a KV head).
+ * Dense and varlen batches.  With rolekv_batch.seqlens_host == NULL every
+ *   sequence has n_max tokens.  Otherwise sequence s has seqlens_host[s]
+ *   tokens (0 <= len <= n_max) and cu_seqlens_dev must hold, on the device, the
+ *   b+1 prefix sums 0, len0, len0+len1, ... (int32).
+ * Tensors.  A rolekv_tensor is a device pointer to bf16 elements plus element
+ *   strides for (layer, sequence, head, token); the last (head-dim) axis is
+ *   contiguous.  Element (l, s, h, t, :) lives at
+ *     ptr + l*s_layer + s*s_seq + h*s_head + t*s_tok            (dense)
+ *     ptr + l*s_layer + (cu[s] + t)*s_tok + h*s_head            (varlen)
+ *   The pointer must be 16-byte aligned and every stride a multiple of 8
+ *   elements; s_layer and s_seq must be multiples of s_tok, and s_head either
+ *   a multiple of s_tok or small enough that all heads fit in one token row
+ *   ((H-1)*s_head + d <= s_tok).  [L][b][H][n][d] and varlen [L][T][H][d]
+ *   contiguous tensors both qualify.
+ * Score arrays (fp32).  Dense: [L][b][Hkv][n_max].  Varlen: [L][Hkv][T],
+ *   sequence s at columns cu[s] .. cu[s+1]-1.
+ * Role arrays (uint8, one label per token, shared by all layers and heads).
+ *   Dense: [b][n_max].  Varlen: [T].
+ * Kept-index arrays (int32).  Sequence s keeps K_s = rolekv_kept_count(len_s,
+ *   B) slots.  Dense: [L][b][Hkv][K], K = rolekv_kept_count(n_max, B).
+ *   Varlen: [L][Hkv][Ktot], sequence s at offset cu_kept[s] = sum of K_s' for
+ *   s' < s.  Kept positions are written in ascending order; when fewer than K_s
+ *   tokens are eligible the tail of the row is -1.
+ * Ownership.  The caller owns every buffer; the library allocates, frees and
+ *   synchronises nothing.  Every call enqueues work on `stream` (a
+ *   cudaStream_t; NULL means the legacy default stream) and returns at once.
+ * Errors.  Argument problems are detected on the host before anything is
+ *   enqueued and return a ROLEKV_ERR_* code; rolekv_last_error() then gives a
+ *   one-line description.  Conditions seen on the device (non-finite scores,
+ *   an out-of-range kept index, a wait that ran out) never trap: they are
+ *   OR-ed into the optional int32 *status_dev word (ROLEKV_STATUS_* bits),
+ *   which the caller clears and reads.
+ */
+#ifndef ROLEKV_H
+#define ROLEKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ROLEKV_OK 0
+#define ROLEKV_ERR_INVALID_ARG 1
+#define ROLEKV_ERR_UNSUPPORTED 2
+#define ROLEKV_ERR_WORKSPACE 3
+#define ROLEKV_ERR_CUDA 4
+
+#define ROLEKV_STATUS_NONFINITE 1   /* a NaN score was seen by the selector    */
+#define ROLEKV_STATUS_BAD_INDEX 2   /* kv_compact met an index >= the length  */
+#define ROLEKV_STATUS_TIMEOUT 4     /* a bounded device wait gave up          */
+
+#define ROLEKV_POLICY_ROLE_QUOTA 0  /* the combined method (Section 4.1)       */
+#define ROLEKV_POLICY_GLOBAL 1      /* plain top-k, optional role ban (Sec. 4) */
+
+#define ROLEKV_MAX_ROLES 8
+#define ROLEKV_SELECT_MAX_N 40960   /* largest sequence role_alloc_select takes */
+
+typedef struct rolekv_tensor {
+  const void* ptr;
+  int64_t s_layer, s_seq, s_head, s_tok;
+} rolekv_tensor;
+
+typedef struct rolekv_batch {
+  int32_t L, b, Hq, Hkv, d;
+  int32_t n_max;
+  const int32_t* seqlens_host;   /* [b] on the host, or NULL (dense)          */
+  const int32_t* cu_seqlens_dev; /* [b+1] on the device, varlen only          */
+} rolekv_batch;
+
+/* Role-conditional allocation parameters (Section 4.1, Algorithm 1).
+ *   alpha[r]   weight of role r (>= 0); alpha[key_role] is replaced by
+ *              alpha_key, the method's one tuned knob (0 bans KEY, 0.02 is the
+ *              paper's safe default).
+ *   budget     B in (0, 1]; a sequence of n tokens keeps ceil(B*n) tokens
+ *              (B is taken to 1e-6 fixed point so the ceiling is exact).
+ *   policy     ROLEKV_POLICY_ROLE_QUOTA: bucket r keeps its share
+ *              alpha_r / sum(alpha of eligible buckets) of the budget, a bucket
+ *              being eligible when alpha_r > 0, it holds tokens and is not
+ *              banned; a bucket whose share reaches its size keeps everything
+ *              and its slack goes to the others in proportion to alpha
+ *              (repeated water-filling), and the integer quotas are floors plus
+ *              largest remainders (ties to the lower role id), so they sum to
+ *              exactly min(ceil(B*n), eligible tokens).
+ *              ROLEKV_POLICY_GLOBAL: one bucket of all non-banned tokens, top
+ *              min(ceil(B*n), eligible) by score (plain H2O / SnapKV top-k;
+ *              with ban_mask it is the counterfactual 'No-X' ban of Section 4).
+ *   ban_mask   bit r set: role r keeps nothing.
+ * Within a bucket the highest scores win and equal scores go to the lower
+ * token index. */
+typedef struct rolekv_select_params {
+  int32_t n_roles;               /* 1 .. ROLEKV_MAX_ROLES                     */
+  float alpha[ROLEKV_MAX_ROLES];
+  int32_t key_role;              /* -1: no override                           */
+  float alpha_key;
+  float budget;
+  int32_t policy;
+  uint32_t ban_mask;
+} rolekv_select_params;
+
+/* Number of kept slots of an n-token sequence at budget B: ceil(B*n) with B in
+ * 1e-6 fixed point; -1 if B is outside (0, 1] or n < 0. */
+int64_t rolekv_kept_count(int64_t n, float budget);
+
+/* Bytes of device workspace snapkv_score / h2o_score / rolekv_compress need for
+ * this batch (op: 0 snapkv_score, 1 h2o_score, 2 rolekv_compress; W the SnapKV
+ * window).  The workspace is caller-owned scratch, 256-byte aligned, reusable
+ * across calls on the same stream; its contents need no initialisation. */
+int rolekv_workspace_size(int op, const rolekv_batch* batch, int32_t W, size_t* bytes);
+
+/* SnapKV windowed score (Section 2; Section 4 'SnapKV mechanism'; Algorithm 1,
+ * windowed mass and pooling steps).  With pool_k == 1 and no scores_prepool
+ * the pre-pool score is written straight to `scores` (no pool kernel).
+ *   q_win   bf16 window queries, [L][b][Hq][W][d] addressed by its strides
+ *           (dense in the sequence axis even for varlen batches); row i of a
+ *           sequence of n tokens is the query at position n - W_eff + i,
+ *           W_eff = min(W, n); rows i >= W_eff are ignored.
+ *   k       bf16 keys of the batch.
+ *   W       window length, a multiple of 8 with W*G <= 256.
+ *   pool_k  odd max-pool width, 1 .. 15 (1 = no pooling).
+ *   scale   softmax scale; <= 0 selects 1/sqrt(d).
+ *   lse_win optional fp32 [L][b][Hq][W]: the natural-log softmax normaliser of
+ *           each window row over its causal keys (the prefill attention's own
+ *           LSE).  NULL: computed here (two passes over K).
+ *   scores  fp32 score array, receives the pooled score s~(t).
+ *   scores_prepool  optional fp32 score array for s(t) before pooling.
+ * s(t) = sum over the G query heads of the KV head and the W_eff window rows of
+ * softmax(scale * q K^T) at key t, causal inside the window; the pool is stride
+ * 1, same length, truncated at the sequence ends.  d must be 64 or 128. */
+int snapkv_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k, int32_t W,
+                 int32_t pool_k, float scale, const float* lse_win, float* scores,
+                 float* scores_prepool, void* workspace, size_t workspace_bytes,
+                 int32_t* status_dev, void* stream);
+
+/* H2O accumulated attention mass (Section 2): s(t) = sum over the G query heads
+ * of the KV head and every causal query position q >= t of p_t(q).
+ *   q       bf16 prefill queries of every position: dense [L][b][Hq][n][d] or
+ *           varlen [L][T][Hq][d], addressed by its strides.
+ *   scores  fp32 score array.  No pooling (the H2O score has none).
+ * d must be 64 or 128 and G <= 8. */
+int h2o_score(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k, float scale,
+              float* scores, void* workspace, size_t workspace_bytes, int32_t* status_dev,
+              void* stream);
+
+/* Role-conditional allocation and per-bucket top-k (Section 4.1, Algorithm 1).
+ *   scores        fp32 score array (pooled SnapKV, H2O, or any score).
+ *   roles         uint8 role array; labels >= n_roles belong to no bucket.
+ *   pool_k        odd width of a max-pool applied to `scores` first (1 = none);
+ *                 lets a caller pass pre-pool SnapKV scores.
+ *   keep_idx      int32 kept-index array (ascending positions, -1 padded).
+ *   keep_mask     optional uint8 array in the score layout: 1 kept, 0 evicted.
+ *   kept_per_role optional int32 [units][n_roles]: kept tokens per role.
+ * Sequences longer than ROLEKV_SELECT_MAX_N are rejected (ERR_UNSUPPORTED). */
+int role_alloc_select(const rolekv_batch* batch, const float* scores, const uint8_t* roles,
+                      const rolekv_select_params* params, int32_t pool_k, int32_t* keep_idx,
+                      uint8_t* keep_mask, int32_t* kept_per_role, int32_t* status_dev,
+                      void* stream);
+
+/* Gather-compaction of the retained rows (Section 6, compacting
+ * implementation): k_out[u][j] = K[u][keep_idx[u][j]] and the same for V, for
+ * every kept slot j; slots holding -1 become zero rows.  k_out / v_out are
+ * dense bf16 [L][b][Hkv][K][d] (varlen: [L][Hkv][Ktot][d]) with the kept-index
+ * layout of `budget`.  d must be a multiple of 8, at most 256. */
+int kv_compact(const rolekv_batch* batch, rolekv_tensor k, rolekv_tensor v,
+               const int32_t* keep_idx, float budget, void* k_out, void* v_out,
+               int32_t* status_dev, void* stream);
+
+/* The whole path in one call: snapkv_score (pre-pool scores kept in the
+ * workspace), role_alloc_select with the pool fused into its load, and
+ * kv_compact.  Arguments as in the calls above; the pooled scores are not
+ * written out. */
+int rolekv_compress(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k,
+                    rolekv_tensor v, int32_t W, int32_t pool_k, float scale,
+                    const float* lse_win, const uint8_t* roles,
+                    const rolekv_select_params* params, int32_t* keep_idx, void* k_out,
+                    void* v_out, int32_t* kept_per_role, void* workspace,
+                    size_t workspace_bytes, int32_t* status_dev, void* stream);
+
+/* Optional per-kernel timing for callers that profile the path.  After this
+ * call every later call made on the same thread records events[i]
+ * (cudaEvent_t, created by the caller) on its stream right after its i-th
+ * kernel launch, for i < n (n <= 8; n = 0 switches it off).  Kernel order:
+ * snapkv_score / rolekv_compress: pass 1 (absent when lse_win is given), the
+ * window normalisers, pass 2, then the pool (snapkv_score with pool_k > 1) or
+ * the selector and the compaction (rolekv_compress); h2o_score: pass 1,
+ * pass 2; role_alloc_select and kv_compact: their one kernel.  The setting
+ * is per thread and holds no device memory. */
+int rolekv_set_stage_events(void* const* events, int32_t n);
+
+/* One-line description of the last error returned on this thread. */
+const char* rolekv_last_error(void);
+
+/* Library version string. */
+const char* rolekv_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ROLEKV_H */

@@ -1,0 +1,102 @@
+// Internal interfaces between the C-ABI layer and the kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "rolekv.h"
+
+namespace rolekv {
+
+enum { kModeSnapKV = 0, kModeH2O = 1 };
+
+// Everything the two attention passes need, passed by value to the kernels.
+struct ScoreArgs {
+  int32_t L, b, G, Hkv, d, n_max;
+  int32_t varlen;
+  int64_t T;                        // packed tokens (varlen score layout)
+  const int32_t* cu_seqlens;        // device, varlen only
+  int32_t mode;                     // kModeSnapKV / kModeH2O
+  int32_t W;                        // SnapKV window
+  int32_t P;                        // positions per query block (SnapKV: W)
+  int32_t nrows;                    // G * P rows in a query block
+  int32_t nrows_pad;                // 128 or 256
+  int32_t n_units;
+  int64_t k_layer, k_seq, k_head, k_tok;
+  int64_t q_layer, q_seq, q_head, q_tok;
+  float c1;                         // softmax scale * log2(e)
+  int32_t chunk_tiles;              // SnapKV: 128-key tiles per CTA
+  int32_t n_chunks;                 // SnapKV: CTAs per unit
+  int32_t nrb_max;                  // H2O: query blocks per unit (largest sequence)
+  float2* partials;                 // SnapKV pass 1: [unit][chunk][256] (max2, sum)
+  float* lse2;                      // [unit][query block][256] log2-domain normalisers
+  float* prepool;                   // score output before pooling
+  int32_t* status;
+};
+
+cudaError_t launch_attn_pass(int pass, int d, const CUtensorMap& kmap, const CUtensorMap& qmap,
+                             const ScoreArgs& a, int grid, cudaStream_t stream);
+cudaError_t launch_snapkv_lse(const ScoreArgs& a, const float* lse_win, cudaStream_t stream);
+cudaError_t launch_maxpool(const ScoreArgs& a, const float* in, float* out, int pool_k,
+                           cudaStream_t stream);
+
+// Selection ------------------------------------------------------------------
+
+struct SelectArgs {
+  int32_t L, b, Hkv, n_max;
+  int32_t varlen;
+  int64_t T;                        // packed tokens
+  int64_t Ktot;                     // packed kept slots (varlen)
+  int32_t K_dense;                  // kept slots per unit (dense)
+  const int32_t* cu_seqlens;
+  int32_t n_units;
+  const float* scores;
+  const uint8_t* roles;
+  int32_t pool_k;
+  int32_t n_roles;
+  int64_t alpha_fx[ROLEKV_MAX_ROLES];   // fixed-point weights, 0 for banned roles
+  int64_t budget_fx;
+  int32_t policy;
+  uint32_t ban_mask;
+  int32_t* keep_idx;
+  uint8_t* keep_mask;
+  int32_t* kept_per_role;
+  int32_t* status;
+};
+
+cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream);
+
+// Compaction -----------------------------------------------------------------
+
+struct CompactArgs {
+  int32_t L, b, Hkv, d, n_max;
+  int32_t varlen;
+  int64_t Ktot;
+  int32_t K_dense;
+  int32_t K_max;                    // widest kept row (grid sizing)
+  int64_t budget_fx;
+  const int32_t* cu_seqlens;
+  int32_t n_units;
+  const uint16_t* k;
+  const uint16_t* v;
+  int64_t k_layer, k_seq, k_head, k_tok;
+  int64_t v_layer, v_seq, v_head, v_tok;
+  const int32_t* keep_idx;
+  uint16_t* k_out;
+  uint16_t* v_out;
+  int32_t* status;
+};
+
+cudaError_t launch_compact(const CompactArgs& a, cudaStream_t stream);
+
+// Shared helpers (host and device) ------------------------------------------
+
+constexpr int64_t kFixedOne = 1000000;
+
+__host__ __device__ inline int64_t kept_slots(int64_t n, int64_t budget_fx) {
+  return (budget_fx * n + kFixedOne - 1) / kFixedOne;
+}
+
+}  // namespace rolekv

@@ -1,0 +1,586 @@
+// C ABI of librolekv (declared in include/rolekv.h): argument checks on the
+// host, TMA descriptors, workspace layout and the kernel launches.  Nothing
+// here allocates device memory or synchronises.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdint>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "internal.h"
+#include "rolekv.h"
+
+namespace rolekv {
+
+size_t select_smem_bytes(int n_max);
+
+namespace {
+
+thread_local char g_err[512] = "no error";
+
+// Optional per-launch timing events of this thread (rolekv_set_stage_events).
+constexpr int kMaxStageEvents = 8;
+thread_local cudaEvent_t g_stage_events[kMaxStageEvents];
+thread_local int g_num_stage_events = 0;
+thread_local int g_stage_cursor = 0;
+
+void stage_begin() { g_stage_cursor = 0; }
+
+// Records the next stage event (if any) after a kernel launch.
+void stage_mark(cudaStream_t stream) {
+  if (g_stage_cursor < g_num_stage_events) cudaEventRecord(g_stage_events[g_stage_cursor], stream);
+  ++g_stage_cursor;
+}
+
+int fail(int code, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return code;
+}
+
+int cuda_fail(cudaError_t e, const char* what) {
+  return fail(ROLEKV_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+constexpr int kRowsMax = 256;
+constexpr int kTileKeys = 128;
+
+int64_t to_fixed(float x) { return static_cast<int64_t>(std::floor(static_cast<double>(x) * 1e6 + 0.5)); }
+
+size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+// ---------------------------------------------------------------- batches --
+
+struct BatchInfo {
+  int L, b, Hq, Hkv, G, d, n_max;
+  bool varlen;
+  int64_t T;
+  int64_t n_units;
+};
+
+int check_batch(const rolekv_batch* bt, BatchInfo* bi) {
+  if (bt == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "batch is NULL");
+  if (bt->L < 1 || bt->b < 1 || bt->Hq < 1 || bt->Hkv < 1 || bt->d < 1 || bt->n_max < 0)
+    return fail(ROLEKV_ERR_INVALID_ARG, "batch sizes must be positive (L=%d b=%d Hq=%d Hkv=%d d=%d n_max=%d)",
+                bt->L, bt->b, bt->Hq, bt->Hkv, bt->d, bt->n_max);
+  if (bt->Hq % bt->Hkv != 0)
+    return fail(ROLEKV_ERR_INVALID_ARG, "Hq=%d is not a multiple of Hkv=%d", bt->Hq, bt->Hkv);
+  bi->L = bt->L;
+  bi->b = bt->b;
+  bi->Hq = bt->Hq;
+  bi->Hkv = bt->Hkv;
+  bi->G = bt->Hq / bt->Hkv;
+  bi->d = bt->d;
+  bi->n_max = bt->n_max;
+  bi->varlen = bt->seqlens_host != nullptr;
+  bi->T = 0;
+  if (bi->varlen) {
+    if (bt->cu_seqlens_dev == nullptr)
+      return fail(ROLEKV_ERR_INVALID_ARG, "varlen batch needs cu_seqlens_dev");
+    for (int s = 0; s < bt->b; ++s) {
+      const int n = bt->seqlens_host[s];
+      if (n < 0 || n > bt->n_max)
+        return fail(ROLEKV_ERR_INVALID_ARG, "seqlens[%d]=%d outside [0, n_max=%d]", s, n, bt->n_max);
+      bi->T += n;
+    }
+    if (bi->T > INT32_MAX) return fail(ROLEKV_ERR_UNSUPPORTED, "more than 2^31-1 packed tokens");
+  } else {
+    bi->T = static_cast<int64_t>(bt->b) * bt->n_max;
+  }
+  bi->n_units = static_cast<int64_t>(bt->L) * bt->b * bt->Hkv;
+  if (bi->n_units > INT32_MAX / 512) return fail(ROLEKV_ERR_UNSUPPORTED, "too many units");
+  return ROLEKV_OK;
+}
+
+// Largest element offset touched by a tensor (exclusive), for the given
+// per-axis extents.
+int64_t tensor_span(const rolekv_tensor& t, int L, int b, int H, int64_t rows, int d, bool packed) {
+  if (packed) return (L - 1) * t.s_layer + (rows - 1) * t.s_tok + (H - 1) * t.s_head + d;
+  return (L - 1) * t.s_layer + (b - 1) * t.s_seq + (H - 1) * t.s_head + (rows - 1) * t.s_tok + d;
+}
+
+int check_tensor(const char* name, const rolekv_tensor& t, int d, int H, bool packed, bool for_tma) {
+  if (t.ptr == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "%s: NULL pointer", name);
+  if (reinterpret_cast<uintptr_t>(t.ptr) % 16 != 0)
+    return fail(ROLEKV_ERR_INVALID_ARG, "%s: pointer not 16-byte aligned", name);
+  if (t.s_layer < 0 || t.s_seq < 0 || t.s_head < 0 || t.s_tok < d)
+    return fail(ROLEKV_ERR_INVALID_ARG, "%s: bad strides", name);
+  if (t.s_layer % 8 || t.s_seq % 8 || t.s_head % 8 || t.s_tok % 8)
+    return fail(ROLEKV_ERR_INVALID_ARG, "%s: strides must be multiples of 8 elements", name);
+  if (for_tma) {
+    if (t.s_layer % t.s_tok || (!packed && t.s_seq % t.s_tok))
+      return fail(ROLEKV_ERR_INVALID_ARG, "%s: layer/sequence strides must be multiples of the token stride", name);
+    if (t.s_head % t.s_tok != 0 && (H - 1) * t.s_head + d > t.s_tok)
+      return fail(ROLEKV_ERR_INVALID_ARG, "%s: heads neither whole token rows nor inside one token row", name);
+  }
+  return ROLEKV_OK;
+}
+
+// ------------------------------------------------------------- tensor maps --
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 2-D bf16 map over the token rows of a tensor: x runs over the s_tok elements
+// of a token row, y over the rows; boxes of 64 x box_rows with the 128-byte
+// swizzle the MMA descriptors expect.
+int make_row_map(CUtensorMap* map, const rolekv_tensor& t, int64_t span, int box_rows) {
+  auto fn = encode_fn();
+  if (fn == nullptr) return fail(ROLEKV_ERR_CUDA, "cuTensorMapEncodeTiled is not available");
+  const int64_t rows = (span + t.s_tok - 1) / t.s_tok;
+  if (rows >= (int64_t(1) << 31)) return fail(ROLEKV_ERR_UNSUPPORTED, "tensor has too many token rows for TMA");
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(t.s_tok), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(t.s_tok) * 2};
+  cuuint32_t box[2] = {64, static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(t.ptr), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(ROLEKV_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
+  return ROLEKV_OK;
+}
+
+int num_sms() {
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      sms = 148;
+  }
+  return sms;
+}
+
+// ------------------------------------------------------------ score plans --
+
+struct ScorePlan {
+  ScoreArgs a;
+  size_t off_partials, off_lse, off_prepool, bytes;
+  int grid1, grid2;
+};
+
+int64_t score_elems(const BatchInfo& bi) {
+  return bi.varlen ? static_cast<int64_t>(bi.L) * bi.Hkv * bi.T : bi.n_units * bi.n_max;
+}
+
+int plan_score(int mode, const BatchInfo& bi, int W, bool need_partials, bool need_prepool,
+               ScorePlan* p) {
+  ScoreArgs& a = p->a;
+  std::memset(&a, 0, sizeof(a));
+  if (bi.d != 64 && bi.d != 128)
+    return fail(ROLEKV_ERR_UNSUPPORTED, "head dim %d (the score kernels take 64 or 128)", bi.d);
+  a.L = bi.L;
+  a.b = bi.b;
+  a.G = bi.G;
+  a.Hkv = bi.Hkv;
+  a.d = bi.d;
+  a.n_max = bi.n_max;
+  a.varlen = bi.varlen;
+  a.T = bi.T;
+  a.mode = mode;
+  a.n_units = static_cast<int32_t>(bi.n_units);
+  if (mode == kModeSnapKV) {
+    if (W < 8 || W % 8 != 0 || W * bi.G > kRowsMax)
+      return fail(ROLEKV_ERR_UNSUPPORTED, "window W=%d must be a multiple of 8 with W*G <= 256 (G=%d)", W, bi.G);
+    a.W = W;
+    a.P = W;
+  } else {
+    if (bi.G > 8) return fail(ROLEKV_ERR_UNSUPPORTED, "H2O takes G <= 8 query heads per KV head (G=%d)", bi.G);
+    a.P = bi.G <= 4 ? 64 : 32;
+  }
+  a.nrows = bi.G * a.P;
+  a.nrows_pad = a.nrows <= 128 ? 128 : 256;
+  const int ntiles = (bi.n_max + kTileKeys - 1) / kTileKeys;
+  if (mode == kModeSnapKV) {
+    a.chunk_tiles = ntiles < 64 ? (ntiles > 0 ? ntiles : 1) : 64;
+    a.n_chunks = (ntiles + a.chunk_tiles - 1) / a.chunk_tiles;
+    if (a.n_chunks < 1) a.n_chunks = 1;
+    p->grid1 = a.n_units * a.n_chunks;
+    p->grid2 = p->grid1;
+    a.nrb_max = 1;
+  } else {
+    a.nrb_max = (bi.n_max + a.P - 1) / a.P;
+    p->grid1 = a.n_units * a.nrb_max;
+    p->grid2 = a.n_units * ntiles;
+  }
+  size_t off = 256;   // first 256 bytes reserved
+  p->off_partials = off;
+  if (need_partials) off += align256(static_cast<size_t>(a.n_units) * a.n_chunks * kRowsMax * 8);
+  p->off_lse = off;
+  off += align256(static_cast<size_t>(a.n_units) * a.nrb_max * kRowsMax * 4);
+  p->off_prepool = off;
+  if (need_prepool) off += align256(static_cast<size_t>(score_elems(bi)) * 4);
+  p->bytes = off;
+  return ROLEKV_OK;
+}
+
+void set_strides(ScoreArgs& a, const rolekv_tensor& k, const rolekv_tensor& q) {
+  a.k_layer = k.s_layer;
+  a.k_seq = k.s_seq;
+  a.k_head = k.s_head;
+  a.k_tok = k.s_tok;
+  a.q_layer = q.s_layer;
+  a.q_seq = q.s_seq;
+  a.q_head = q.s_head;
+  a.q_tok = q.s_tok;
+}
+
+int bind_workspace(ScorePlan& p, void* ws, size_t ws_bytes) {
+  if (ws == nullptr || ws_bytes < p.bytes)
+    return fail(ROLEKV_ERR_WORKSPACE, "workspace of %zu bytes given, %zu needed", ws_bytes, p.bytes);
+  if (reinterpret_cast<uintptr_t>(ws) % 256 != 0)
+    return fail(ROLEKV_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+  uint8_t* base = static_cast<uint8_t*>(ws);
+  p.a.partials = reinterpret_cast<float2*>(base + p.off_partials);
+  p.a.lse2 = reinterpret_cast<float*>(base + p.off_lse);
+  return ROLEKV_OK;
+}
+
+// SnapKV scores: pass 1 + normalisers (or the caller's LSE) + pass 2, the
+// pre-pool scores going to `prepool`.
+int run_snapkv(const BatchInfo& bi, const int32_t* cu_seqlens, const rolekv_tensor& q_win,
+               const rolekv_tensor& k, int W, float scale, const float* lse_win, float* prepool,
+               ScorePlan& p, int32_t* status, cudaStream_t stream) {
+  ScoreArgs& a = p.a;
+  set_strides(a, k, q_win);
+  a.c1 = (scale > 0.f ? scale : 1.0f / std::sqrt(static_cast<float>(bi.d))) * 1.4426950408889634f;
+  a.prepool = prepool;
+  a.status = status;
+  a.cu_seqlens = cu_seqlens;
+  CUtensorMap kmap, qmap;
+  int rc = make_row_map(&kmap, k,
+                        tensor_span(k, bi.L, bi.b, bi.Hkv, bi.varlen ? bi.T : bi.n_max, bi.d, bi.varlen),
+                        kTileKeys);
+  if (rc) return rc;
+  rc = make_row_map(&qmap, q_win, tensor_span(q_win, bi.L, bi.b, bi.Hq, W, bi.d, false), W);
+  if (rc) return rc;
+  cudaError_t e;
+  if (lse_win == nullptr) {
+    e = launch_attn_pass(0, bi.d, kmap, qmap, a, p.grid1, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "snapkv pass 1");
+    stage_mark(stream);
+  }
+  e = launch_snapkv_lse(a, lse_win, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "snapkv normalisers");
+  stage_mark(stream);
+  e = launch_attn_pass(1, bi.d, kmap, qmap, a, p.grid2, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "snapkv pass 2");
+  stage_mark(stream);
+  return ROLEKV_OK;
+}
+
+void fill_compact(const BatchInfo& bi, const int32_t* cu_seqlens, int64_t budget_fx,
+                  const int32_t* seqlens_host, const rolekv_tensor& k, const rolekv_tensor& v,
+                  const int32_t* keep_idx, void* k_out, void* v_out, int32_t* status,
+                  CompactArgs* a) {
+  std::memset(a, 0, sizeof(*a));
+  a->L = bi.L;
+  a->b = bi.b;
+  a->Hkv = bi.Hkv;
+  a->d = bi.d;
+  a->n_max = bi.n_max;
+  a->varlen = bi.varlen;
+  a->budget_fx = budget_fx;
+  a->K_dense = static_cast<int32_t>(kept_slots(bi.n_max, budget_fx));
+  a->K_max = a->K_dense;
+  a->Ktot = 0;
+  if (bi.varlen)
+    for (int s = 0; s < bi.b; ++s) a->Ktot += kept_slots(seqlens_host[s], budget_fx);
+  a->cu_seqlens = cu_seqlens;
+  a->n_units = static_cast<int32_t>(bi.n_units);
+  a->k = static_cast<const uint16_t*>(k.ptr);
+  a->v = static_cast<const uint16_t*>(v.ptr);
+  a->k_layer = k.s_layer;
+  a->k_seq = k.s_seq;
+  a->k_head = k.s_head;
+  a->k_tok = k.s_tok;
+  a->v_layer = v.s_layer;
+  a->v_seq = v.s_seq;
+  a->v_head = v.s_head;
+  a->v_tok = v.s_tok;
+  a->keep_idx = keep_idx;
+  a->k_out = static_cast<uint16_t*>(k_out);
+  a->v_out = static_cast<uint16_t*>(v_out);
+  a->status = status;
+}
+
+int check_compact_args(const BatchInfo& bi, const rolekv_tensor& k, const rolekv_tensor& v,
+                       const int32_t* keep_idx, void* k_out, void* v_out) {
+  if (bi.d < 8 || bi.d > 256 || (bi.d & (bi.d - 1)) != 0)
+    return fail(ROLEKV_ERR_UNSUPPORTED, "kv_compact takes d a power of two in 8..256 (d=%d)", bi.d);
+  if (keep_idx == nullptr || k_out == nullptr || v_out == nullptr)
+    return fail(ROLEKV_ERR_INVALID_ARG, "keep_idx, k_out and v_out are required");
+  if (reinterpret_cast<uintptr_t>(k_out) % 16 || reinterpret_cast<uintptr_t>(v_out) % 16)
+    return fail(ROLEKV_ERR_INVALID_ARG, "k_out/v_out must be 16-byte aligned");
+  int rc;
+  if ((rc = check_tensor("k", k, bi.d, bi.Hkv, bi.varlen, false))) return rc;
+  if ((rc = check_tensor("v", v, bi.d, bi.Hkv, bi.varlen, false))) return rc;
+  return ROLEKV_OK;
+}
+
+// ---------------------------------------------------------- select / compact --
+
+int fill_select(const BatchInfo& bi, const rolekv_batch* bt, const rolekv_select_params* sp,
+                SelectArgs* a) {
+  std::memset(a, 0, sizeof(*a));
+  if (sp == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "select params are NULL");
+  if (sp->n_roles < 1 || sp->n_roles > ROLEKV_MAX_ROLES)
+    return fail(ROLEKV_ERR_UNSUPPORTED, "n_roles=%d outside 1..%d", sp->n_roles, ROLEKV_MAX_ROLES);
+  if (!(sp->budget > 0.f) || sp->budget > 1.f)
+    return fail(ROLEKV_ERR_INVALID_ARG, "budget %g outside (0, 1]", static_cast<double>(sp->budget));
+  if (sp->policy != ROLEKV_POLICY_ROLE_QUOTA && sp->policy != ROLEKV_POLICY_GLOBAL)
+    return fail(ROLEKV_ERR_INVALID_ARG, "unknown policy %d", sp->policy);
+  if (sp->key_role >= sp->n_roles) return fail(ROLEKV_ERR_INVALID_ARG, "key_role %d >= n_roles", sp->key_role);
+  if (bi.n_max > ROLEKV_SELECT_MAX_N)
+    return fail(ROLEKV_ERR_UNSUPPORTED, "n_max=%d exceeds the %d tokens the selector holds", bi.n_max,
+                ROLEKV_SELECT_MAX_N);
+  a->L = bi.L;
+  a->b = bi.b;
+  a->Hkv = bi.Hkv;
+  a->n_max = bi.n_max;
+  a->varlen = bi.varlen;
+  a->T = bi.T;
+  a->cu_seqlens = bt->cu_seqlens_dev;
+  a->n_units = static_cast<int32_t>(bi.n_units);
+  a->n_roles = sp->n_roles;
+  a->budget_fx = to_fixed(sp->budget);
+  a->policy = sp->policy;
+  a->ban_mask = sp->ban_mask;
+  for (int r = 0; r < ROLEKV_MAX_ROLES; ++r) {
+    float al = r < sp->n_roles ? sp->alpha[r] : 0.f;
+    if (r == sp->key_role) al = sp->alpha_key;
+    if (!(al >= 0.f) || !std::isfinite(al))
+      return fail(ROLEKV_ERR_INVALID_ARG, "alpha[%d]=%g must be finite and >= 0", r, static_cast<double>(al));
+    a->alpha_fx[r] = ((sp->ban_mask >> r) & 1u) ? 0 : to_fixed(al);
+  }
+  a->K_dense = static_cast<int32_t>(kept_slots(bi.n_max, a->budget_fx));
+  a->Ktot = 0;
+  if (bi.varlen)
+    for (int s = 0; s < bi.b; ++s) a->Ktot += kept_slots(bt->seqlens_host[s], a->budget_fx);
+  return ROLEKV_OK;
+}
+
+}  // namespace
+}  // namespace rolekv
+
+using namespace rolekv;
+
+extern "C" {
+
+int64_t rolekv_kept_count(int64_t n, float budget) {
+  if (n < 0 || !(budget > 0.f) || budget > 1.f) return -1;
+  return kept_slots(n, to_fixed(budget));
+}
+
+const char* rolekv_last_error(void) { return g_err; }
+
+const char* rolekv_version(void) { return "rolekv 0.1 (sm_103a)"; }
+
+int rolekv_workspace_size(int op, const rolekv_batch* batch, int32_t W, size_t* bytes) {
+  if (bytes == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "bytes is NULL");
+  BatchInfo bi;
+  int rc = check_batch(batch, &bi);
+  if (rc) return rc;
+  ScorePlan p;
+  switch (op) {
+    case 0: rc = plan_score(kModeSnapKV, bi, W, true, true, &p); break;
+    case 1: rc = plan_score(kModeH2O, bi, 0, false, false, &p); break;
+    case 2: rc = plan_score(kModeSnapKV, bi, W, true, true, &p); break;
+    default: return fail(ROLEKV_ERR_INVALID_ARG, "unknown op %d", op);
+  }
+  if (rc) return rc;
+  *bytes = p.bytes;
+  return ROLEKV_OK;
+}
+
+int snapkv_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k, int32_t W,
+                 int32_t pool_k, float scale, const float* lse_win, float* scores,
+                 float* scores_prepool, void* workspace, size_t workspace_bytes,
+                 int32_t* status_dev, void* stream) {
+  BatchInfo bi;
+  int rc = check_batch(batch, &bi);
+  if (rc) return rc;
+  if (pool_k < 1 || pool_k > 15 || pool_k % 2 == 0)
+    return fail(ROLEKV_ERR_UNSUPPORTED, "pool_k=%d must be odd, 1..15", pool_k);
+  if (scores == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "scores is NULL");
+  ScorePlan p;
+  rc = plan_score(kModeSnapKV, bi, W, lse_win == nullptr, scores_prepool == nullptr, &p);
+  if (rc) return rc;
+  if ((rc = check_tensor("q_win", q_win, bi.d, bi.Hq, false, true))) return rc;
+  if ((rc = check_tensor("k", k, bi.d, bi.Hkv, bi.varlen, true))) return rc;
+  if ((rc = bind_workspace(p, workspace, workspace_bytes))) return rc;
+  if (bi.n_max == 0) return ROLEKV_OK;
+  // Without pooling, pass 2 writes the scores directly.
+  float* pre = scores_prepool ? scores_prepool
+               : pool_k == 1  ? scores
+                              : reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) + p.off_prepool);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  stage_begin();
+  rc = run_snapkv(bi, batch->cu_seqlens_dev, q_win, k, W, scale, lse_win, pre, p, status_dev, st);
+  if (rc) return rc;
+  const ScoreArgs& a = p.a;
+  if (pre == scores) return ROLEKV_OK;
+  cudaError_t e = launch_maxpool(a, pre, scores, pool_k, st);
+  if (e != cudaSuccess) return cuda_fail(e, "max-pool");
+  stage_mark(st);
+  return ROLEKV_OK;
+}
+
+int h2o_score(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k, float scale,
+              float* scores, void* workspace, size_t workspace_bytes, int32_t* status_dev,
+              void* stream) {
+  BatchInfo bi;
+  int rc = check_batch(batch, &bi);
+  if (rc) return rc;
+  if (scores == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "scores is NULL");
+  ScorePlan p;
+  rc = plan_score(kModeH2O, bi, 0, false, false, &p);
+  if (rc) return rc;
+  if ((rc = check_tensor("q", q, bi.d, bi.Hq, bi.varlen, true))) return rc;
+  if ((rc = check_tensor("k", k, bi.d, bi.Hkv, bi.varlen, true))) return rc;
+  if ((rc = bind_workspace(p, workspace, workspace_bytes))) return rc;
+  if (bi.n_max == 0) return ROLEKV_OK;
+  ScoreArgs& a = p.a;
+  set_strides(a, k, q);
+  a.cu_seqlens = batch->cu_seqlens_dev;
+  a.c1 = (scale > 0.f ? scale : 1.0f / std::sqrt(static_cast<float>(bi.d))) * 1.4426950408889634f;
+  a.prepool = scores;
+  a.status = status_dev;
+  CUtensorMap kmap, qmap;
+  const int64_t rows = bi.varlen ? bi.T : bi.n_max;
+  rc = make_row_map(&kmap, k, tensor_span(k, bi.L, bi.b, bi.Hkv, rows, bi.d, bi.varlen), kTileKeys);
+  if (rc) return rc;
+  rc = make_row_map(&qmap, q, tensor_span(q, bi.L, bi.b, bi.Hq, rows, bi.d, bi.varlen), a.P);
+  if (rc) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  stage_begin();
+  cudaError_t e = launch_attn_pass(0, bi.d, kmap, qmap, a, p.grid1, st);
+  if (e != cudaSuccess) return cuda_fail(e, "h2o pass 1");
+  stage_mark(st);
+  e = launch_attn_pass(1, bi.d, kmap, qmap, a, p.grid2, st);
+  if (e != cudaSuccess) return cuda_fail(e, "h2o pass 2");
+  stage_mark(st);
+  return ROLEKV_OK;
+}
+
+int role_alloc_select(const rolekv_batch* batch, const float* scores, const uint8_t* roles,
+                      const rolekv_select_params* params, int32_t pool_k, int32_t* keep_idx,
+                      uint8_t* keep_mask, int32_t* kept_per_role, int32_t* status_dev,
+                      void* stream) {
+  BatchInfo bi;
+  int rc = check_batch(batch, &bi);
+  if (rc) return rc;
+  if (scores == nullptr || roles == nullptr || keep_idx == nullptr)
+    return fail(ROLEKV_ERR_INVALID_ARG, "scores, roles and keep_idx are required");
+  if (pool_k < 1 || pool_k > 15 || pool_k % 2 == 0)
+    return fail(ROLEKV_ERR_UNSUPPORTED, "pool_k=%d must be odd, 1..15", pool_k);
+  SelectArgs a;
+  if ((rc = fill_select(bi, batch, params, &a))) return rc;
+  a.scores = scores;
+  a.roles = roles;
+  a.pool_k = pool_k;
+  a.keep_idx = keep_idx;
+  a.keep_mask = keep_mask;
+  a.kept_per_role = kept_per_role;
+  a.status = status_dev;
+  if (bi.n_max == 0) return ROLEKV_OK;
+  stage_begin();
+  cudaError_t e = launch_select(a, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "role_alloc_select");
+  stage_mark(static_cast<cudaStream_t>(stream));
+  return ROLEKV_OK;
+}
+
+int kv_compact(const rolekv_batch* batch, rolekv_tensor k, rolekv_tensor v,
+               const int32_t* keep_idx, float budget, void* k_out, void* v_out,
+               int32_t* status_dev, void* stream) {
+  BatchInfo bi;
+  int rc = check_batch(batch, &bi);
+  if (rc) return rc;
+  if (!(budget > 0.f) || budget > 1.f)
+    return fail(ROLEKV_ERR_INVALID_ARG, "budget %g outside (0, 1]", static_cast<double>(budget));
+  if ((rc = check_compact_args(bi, k, v, keep_idx, k_out, v_out))) return rc;
+  CompactArgs a;
+  fill_compact(bi, batch->cu_seqlens_dev, to_fixed(budget), batch->seqlens_host, k, v, keep_idx,
+               k_out, v_out, status_dev, &a);
+  if (bi.n_max == 0) return ROLEKV_OK;
+  stage_begin();
+  cudaError_t e = launch_compact(a, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "kv_compact");
+  stage_mark(static_cast<cudaStream_t>(stream));
+  return ROLEKV_OK;
+}
+
+int rolekv_compress(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k,
+                    rolekv_tensor v, int32_t W, int32_t pool_k, float scale,
+                    const float* lse_win, const uint8_t* roles,
+                    const rolekv_select_params* params, int32_t* keep_idx, void* k_out,
+                    void* v_out, int32_t* kept_per_role, void* workspace,
+                    size_t workspace_bytes, int32_t* status_dev, void* stream) {
+  BatchInfo bi;
+  int rc = check_batch(batch, &bi);
+  if (rc) return rc;
+  if (pool_k < 1 || pool_k > 15 || pool_k % 2 == 0)
+    return fail(ROLEKV_ERR_UNSUPPORTED, "pool_k=%d must be odd, 1..15", pool_k);
+  ScorePlan p;
+  rc = plan_score(kModeSnapKV, bi, W, true, true, &p);
+  if (rc) return rc;
+  SelectArgs sa;
+  if ((rc = fill_select(bi, batch, params, &sa))) return rc;
+  if (roles == nullptr || keep_idx == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "roles and keep_idx are required");
+  if ((rc = check_tensor("q_win", q_win, bi.d, bi.Hq, false, true))) return rc;
+  if ((rc = check_tensor("k", k, bi.d, bi.Hkv, bi.varlen, true))) return rc;
+  if ((rc = check_compact_args(bi, k, v, keep_idx, k_out, v_out))) return rc;
+  if ((rc = bind_workspace(p, workspace, workspace_bytes))) return rc;
+  if (bi.n_max == 0) return ROLEKV_OK;
+  float* pre = reinterpret_cast<float*>(static_cast<uint8_t*>(workspace) + p.off_prepool);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  stage_begin();
+  rc = run_snapkv(bi, batch->cu_seqlens_dev, q_win, k, W, scale, lse_win, pre, p, status_dev, st);
+  if (rc) return rc;
+  sa.scores = pre;
+  sa.roles = roles;
+  sa.pool_k = pool_k;
+  sa.keep_idx = keep_idx;
+  sa.keep_mask = nullptr;
+  sa.kept_per_role = kept_per_role;
+  sa.status = status_dev;
+  cudaError_t e = launch_select(sa, st);
+  if (e != cudaSuccess) return cuda_fail(e, "role_alloc_select");
+  stage_mark(st);
+  CompactArgs ca;
+  fill_compact(bi, batch->cu_seqlens_dev, sa.budget_fx, batch->seqlens_host, k, v, keep_idx, k_out,
+               v_out, status_dev, &ca);
+  e = launch_compact(ca, st);
+  if (e != cudaSuccess) return cuda_fail(e, "kv_compact");
+  stage_mark(st);
+  return ROLEKV_OK;
+}
+
+int rolekv_set_stage_events(void* const* events, int32_t n) {
+  if (n < 0 || n > kMaxStageEvents || (n > 0 && events == nullptr))
+    return fail(ROLEKV_ERR_INVALID_ARG, "0..%d stage events", kMaxStageEvents);
+  for (int i = 0; i < n; ++i) g_stage_events[i] = static_cast<cudaEvent_t>(events[i]);
+  g_num_stage_events = n;
+  return ROLEKV_OK;
+}
+
+}  // extern "C"

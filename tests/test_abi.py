@@ -1,0 +1,120 @@
+"""The C ABI on the CPU: the library loads, exports every function that
+include/rolekv.h declares, and rejects bad arguments on the host before
+touching the GPU."""
+
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import rolekv_oracle as O
+from paper_2607_13205_gb300 import build as B
+from paper_2607_13205_gb300 import rolekv as R
+
+HEADER = os.path.join(B.ROOT, "include", "rolekv.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not os.path.exists(B.LIB_PATH):
+        B.build()
+    return R.lib()
+
+
+def _declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    names = re.findall(r"^\s*(?:const\s+)?[A-Za-z_][A-Za-z0-9_]*\s*\*?\s*([A-Za-z_][A-Za-z0-9_]*)\s*\(",
+                       text, flags=re.M)
+    return sorted(set(n for n in names if n not in ("if", "while", "for", "sizeof")))
+
+
+def test_header_declares_the_four_calls():
+    names = _declared_functions()
+    for n in ("snapkv_score", "h2o_score", "role_alloc_select", "kv_compact"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = _declared_functions()
+    assert len(names) >= 8
+    for n in names:
+        assert hasattr(lib, n), f"{n} declared in rolekv.h but not exported"
+
+
+def test_kept_count_matches_oracle(lib):
+    for n in (0, 1, 7, 100, 2048, 8192, 32768, 40960, 123457):
+        for b in (0.05, 0.1, 0.2, 0.3, 0.5, 0.75, 1.0, 0.333):
+            assert R.kept_count(n, b) == O.kept_count(n, b), (n, b)
+    assert R.kept_count(10, 0.0) == -1
+    assert R.kept_count(10, 1.5) == -1
+    assert R.kept_count(-1, 0.5) == -1
+
+
+def _batch(**kw):
+    d = dict(L=2, b=3, Hq=8, Hkv=2, d=128, n_max=1000)
+    d.update(kw)
+    return R.BatchDesc(d["L"], d["b"], d["Hq"], d["Hkv"], d["d"], d["n_max"], None, None)
+
+
+def _ws(op, batch, W):
+    out = ctypes.c_size_t(0)
+    rc = R.lib().rolekv_workspace_size(op, ctypes.byref(batch), W, ctypes.byref(out))
+    return rc, out.value
+
+
+def test_workspace_size(lib):
+    rc, sz = _ws(0, _batch(), 32)
+    assert rc == 0 and sz >= 2 * 3 * 2 * 1000 * 4
+    rc, sz_h2o = _ws(1, _batch(), 0)
+    assert rc == 0 and sz_h2o > 0
+    assert _ws(0, _batch(), 12)[0] == R.ERR_UNSUPPORTED        # W not a multiple of 8
+    assert _ws(0, _batch(Hq=16, Hkv=2), 64)[0] == R.ERR_UNSUPPORTED   # W*G > 256
+    assert _ws(0, _batch(d=96), 32)[0] == R.ERR_UNSUPPORTED
+    assert _ws(0, _batch(Hq=7, Hkv=2), 32)[0] == R.ERR_INVALID_ARG
+    assert _ws(1, _batch(Hq=18, Hkv=2), 0)[0] == R.ERR_UNSUPPORTED   # H2O G > 8
+    assert _ws(9, _batch(), 32)[0] == R.ERR_INVALID_ARG
+
+
+def test_host_rejects_bad_arguments(lib):
+    b = _batch()
+    t = R.Tensor(16, 0, 0, 0, 128)        # fake, never dereferenced: checks fail first
+    f = ctypes.c_void_p(256)
+    rc = lib.snapkv_score(ctypes.byref(b), t, t, 32, 4, 0.0, None, f, None, f, 1 << 30, None, None)
+    assert rc == R.ERR_UNSUPPORTED                                      # even pool width
+    rc = lib.snapkv_score(ctypes.byref(b), t, t, 32, 7, 0.0, None, None, None, f, 1 << 30, None, None)
+    assert rc == R.ERR_INVALID_ARG                                      # no output
+    bad = R.Tensor(24, 0, 0, 0, 128)       # misaligned pointer
+    rc = lib.snapkv_score(ctypes.byref(b), bad, t, 32, 7, 0.0, None, f, None, f, 1 << 30, None, None)
+    assert rc == R.ERR_INVALID_ARG
+    assert b"aligned" in lib.rolekv_last_error()
+    p = R.select_params(0.1, [0.25, 0.0, 0.7, 0.05])
+    rc = lib.role_alloc_select(ctypes.byref(b), f, f, ctypes.byref(p), 2, f, None, None, None, None)
+    assert rc == R.ERR_UNSUPPORTED                                      # even pool width
+    p_bad = R.select_params(1.5, [0.25, 0.0, 0.7, 0.05])
+    rc = lib.role_alloc_select(ctypes.byref(b), f, f, ctypes.byref(p_bad), 1, f, None, None, None, None)
+    assert rc == R.ERR_INVALID_ARG
+    p_neg = R.select_params(0.1, [0.25, 0.0, -0.7, 0.05])
+    rc = lib.role_alloc_select(ctypes.byref(b), f, f, ctypes.byref(p_neg), 1, f, None, None, None, None)
+    assert rc == R.ERR_INVALID_ARG
+    big = _batch(n_max=R.SELECT_MAX_N + 1)
+    rc = lib.role_alloc_select(ctypes.byref(big), f, f, ctypes.byref(p), 1, f, None, None, None, None)
+    assert rc == R.ERR_UNSUPPORTED
+    rc = lib.kv_compact(ctypes.byref(_batch(d=96)), t, t, f, 0.1, f, f, None, None)
+    assert rc == R.ERR_UNSUPPORTED
+    rc = lib.kv_compact(ctypes.byref(b), t, t, f, 0.1, None, f, None, None)
+    assert rc == R.ERR_INVALID_ARG
+    lens = (ctypes.c_int32 * 3)(10, 2000, 5)
+    vb = R.BatchDesc(2, 3, 8, 2, 128, 1000, lens, ctypes.c_void_p(64))
+    rc = lib.kv_compact(ctypes.byref(vb), t, t, f, 0.1, f, f, None, None)
+    assert rc == R.ERR_INVALID_ARG                                      # length > n_max
+    assert b"seqlens" in lib.rolekv_last_error()
+
+
+def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
+    monkeypatch.setattr(R, "_LIB_PATH", str(tmp_path / "missing.so"))
+    monkeypatch.setattr(R, "_lib", None)
+    with pytest.raises(RuntimeError, match="missing"):
+        R.kept_count(10, 0.5)

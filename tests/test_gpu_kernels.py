@@ -1,0 +1,299 @@
+"""GPU parity: every entry point of librolekv against the fp64 oracle, through
+the C ABI, on seeded synthetic inputs (sizes that span several tiles, a
+ragged tail, varlen batches with empty and short sequences)."""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import rolekv_oracle as O
+from paper_2607_13205_gb300 import inputs as I
+from paper_2607_13205_gb300 import rolekv as R
+from tests.gpu_helpers import assert_scores_close, check_index_sets, lib_batch, oracle_batch
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda"
+
+
+def _w(name="tiny", **kw):
+    return I.WORKLOADS[name].scaled(**kw)
+
+
+SNAPKV_CASES = {
+    "tiny_d64": _w("tiny"),
+    "ragged_tail_g4w32": _w("llama8b", L=2, b=2, Hq=8, Hkv=2, n=1000),
+    "two_row_tiles_w64_multichunk": _w("long", L=1, b=1, Hq=8, Hkv=2, n=8500),
+    "g7_224_rows": _w("ragged", L=1, b=2, Hq=14, Hkv=2, n=2100, seqlens=None),
+    "varlen_short_empty": _w("ragged", L=2, b=5, Hq=8, Hkv=2, n=2049, seqlens=(1000, 17, 0, 300, 2049)),
+    "varlen_g7": _w("ragged", L=1, b=3, Hq=14, Hkv=2, n=1500, seqlens=(1500, 31, 640)),
+}
+
+
+def _snapkv_inputs(w, seed=0):
+    roles = I.workload_roles(w, seed)
+    K, V = I.make_kv(w, roles, seed, device=DEV)
+    qw = I.make_q_window(w, seed, device=DEV)
+    return roles, K, V, qw
+
+
+@pytest.mark.parametrize("case", list(SNAPKV_CASES))
+def test_snapkv_score_matches_oracle(case):
+    w = SNAPKV_CASES[case]
+    roles, K, V, qw = _snapkv_inputs(w)
+    batch = lib_batch(w, DEV)
+    scores = torch.full(batch.score_shape(), -1.0, dtype=torch.float32, device=DEV)
+    pre = torch.full_like(scores, -1.0)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    R.snapkv_score(batch, qw, K, w.W, w.pool_k, scores, scores_prepool=pre, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    ob = oracle_batch(w)
+    ref = O.snapkv_batch(ob, I.bf16_bits(qw), I.bf16_bits(K), w.W, w.pool_k)
+    got, gpre = scores.cpu().numpy(), pre.cpu().numpy()
+    for u, (rpre, rpool) in ref.items():
+        assert_scores_close(ob.score_view(gpre, u), rpre, f"{case} unit {u} pre-pool")
+        assert_scores_close(ob.score_view(got, u), rpool, f"{case} unit {u} pooled")
+        n = rpre.size
+        if n:
+            assert abs(ob.score_view(gpre, u).astype(np.float64).sum() - min(w.W, n) * w.G) < 1e-3 * min(w.W, n) * w.G
+
+
+def test_snapkv_with_supplied_lse():
+    """Single pass with the window rows' normalisers given (natural log)."""
+    w = SNAPKV_CASES["varlen_short_empty"]
+    roles, K, V, qw = _snapkv_inputs(w, seed=3)
+    ob = oracle_batch(w)
+    kb, qb = I.bf16_bits(K), I.bf16_bits(qw)
+    lse = np.zeros((w.L, w.b, w.Hq, w.W), dtype=np.float32)
+    scale = 1.0 / np.sqrt(w.d)
+    for u in range(ob.n_units):
+        l, s, h = ob.unit(u)
+        k = O.bf16_to_f64(ob.kv_rows(kb, u))
+        n = k.shape[0]
+        if n == 0:
+            continue
+        w_eff = min(w.W, n)
+        for g in range(w.G):
+            q = O.bf16_to_f64(qb[l, s, h * w.G + g, :w_eff])
+            logits = scale * (q @ k.T)
+            for i in range(w_eff):
+                row = logits[i, :n - w_eff + i + 1]
+                m = row.max()
+                lse[l, s, h * w.G + g, i] = m + np.log(np.exp(row - m).sum())
+    batch = lib_batch(w, DEV)
+    scores = torch.empty(batch.score_shape(), dtype=torch.float32, device=DEV)
+    R.snapkv_score(batch, qw, K, w.W, w.pool_k, scores, lse_win=torch.as_tensor(lse, device=DEV))
+    torch.cuda.synchronize()
+    ref = O.snapkv_batch(ob, qb, kb, w.W, w.pool_k)
+    got = scores.cpu().numpy()
+    for u, (_, rpool) in ref.items():
+        # the normaliser is rounded to fp32 once more here: 2e-3 covers it
+        g = ob.score_view(got, u).astype(np.float64)
+        assert np.all(np.abs(g - rpool) <= 2e-3 * np.abs(rpool) + 1e-20), f"unit {u}"
+
+
+H2O_CASES = {
+    "dense_g4_ragged": _w("h2o", L=1, b=2, Hq=8, Hkv=2, n=700),
+    "dense_g7": _w("h2o", L=1, b=1, Hq=14, Hkv=2, n=450),
+    "varlen": _w("h2o", L=2, b=4, Hq=8, Hkv=2, n=300, seqlens=(300, 129, 0, 64)),
+    "d64": _w("h2o", L=1, b=1, Hq=8, Hkv=2, d=64, n=520),
+}
+
+
+@pytest.mark.parametrize("case", list(H2O_CASES))
+def test_h2o_score_matches_oracle(case):
+    w = H2O_CASES[case]
+    roles = I.workload_roles(w, 1)
+    K, _ = I.make_kv(w, roles, 1, device=DEV, with_v=False)
+    Q = I.make_q_full(w, 1, device=DEV)
+    batch = lib_batch(w, DEV)
+    scores = torch.full(batch.score_shape(), -1.0, dtype=torch.float32, device=DEV)
+    R.h2o_score(batch, Q, K, scores)
+    torch.cuda.synchronize()
+    ob = oracle_batch(w)
+    ref = O.h2o_batch(ob, I.bf16_bits(Q), I.bf16_bits(K))
+    got = scores.cpu().numpy()
+    for u, s in ref.items():
+        assert_scores_close(ob.score_view(got, u), s, f"{case} unit {u}")
+        if s.size:
+            assert abs(ob.score_view(got, u).astype(np.float64).sum() - s.size * w.G) < 1e-3 * s.size * w.G
+
+
+# ------------------------------------------------------------------ selection
+
+def _tied_scores(shape, seed):
+    g = torch.Generator().manual_seed(seed)
+    # coarse values create many exact ties, plateaus like a max-pool's
+    return (torch.randint(0, 64, shape, generator=g).float() / 8.0).to(DEV)
+
+
+SELECT_CASES = [
+    # (name, workload, budget, alpha_key, policy, ban_mask, pool_k)
+    ("combined_b05", _w("llama8b", L=2, b=2, Hq=8, Hkv=2, n=5000), 0.05, 0.0, 0, 0, 1),
+    ("combined_b10_pool7", _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=5000), 0.10, 0.02, 0, 0, 7),
+    ("combined_b50", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=3001), 0.50, 0.0, 0, 0, 1),
+    ("full_budget", _w("llama8b", L=1, b=1, Hq=4, Hkv=1, n=777), 1.0, 0.0, 0, 0, 3),
+    ("global_no_key", _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=4000), 0.30, 0.0, 1, 1 << I.ROLE_KEY, 1),
+    ("global_plain", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=4000), 0.20, 0.0, 1, 0, 5),
+    ("varlen", _w("ragged", L=2, b=4, Hq=8, Hkv=2, n=3000, seqlens=(3000, 0, 5, 1200)), 0.10, 0.0, 0, 0, 7),
+    ("max_n", _w("long", L=1, b=1, Hq=4, Hkv=1, n=R.SELECT_MAX_N), 0.10, 0.0, 0, 0, 7),
+]
+
+
+@pytest.mark.parametrize("case", SELECT_CASES, ids=[c[0] for c in SELECT_CASES])
+def test_role_alloc_select_bit_exact(case):
+    name, w, B, akey, policy, ban, pool_k = case
+    roles_np = I.workload_roles(w, 2)
+    batch = lib_batch(w, DEV)
+    scores = _tied_scores(batch.score_shape(), 5)
+    roles = torch.as_tensor(roles_np, device=DEV)
+    params = R.select_params(B, I.PAPER_ALPHA, alpha_key=akey, key_role=I.ROLE_KEY, policy=policy,
+                             ban_mask=ban)
+    keep = torch.full(batch.kept_shape(B), -7, dtype=torch.int32, device=DEV)
+    mask = torch.full(batch.score_shape(), 9, dtype=torch.uint8, device=DEV)
+    per_role = torch.full((batch.n_units, I.N_ROLES), -1, dtype=torch.int32, device=DEV)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    R.role_alloc_select(batch, scores, roles, params, keep, pool_k=pool_k, keep_mask=mask,
+                        kept_per_role=per_role, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    ob = oracle_batch(w)
+    sc = scores.cpu().numpy()
+    unit_scores = {}
+    for u in range(ob.n_units):
+        s = ob.score_view(sc, u).astype(np.float64)
+        unit_scores[u] = O.maxpool1d(s, pool_k) if s.size else s
+    ref = O.select_batch(ob, unit_scores, roles_np, I.N_ROLES, I.PAPER_ALPHA, I.ROLE_KEY, akey, B,
+                         policy, ban)
+    cu_kept = ob.kept_offsets(B)
+    keep_np, mask_np, pr = keep.cpu().numpy(), mask.cpu().numpy(), per_role.cpu().numpy()
+    for u, (idx, per) in ref.items():
+        l, s, h = ob.unit(u)
+        if ob.varlen:
+            row = keep_np[l, h, cu_kept[s]:cu_kept[s + 1]]
+        else:
+            row = keep_np.reshape(ob.n_units, -1)[u]
+        assert np.array_equal(row, idx), f"{name} unit {u}"
+        assert list(pr[u]) == per, f"{name} unit {u} per-role counts"
+        m = ob.score_view(mask_np, u)
+        expect = np.zeros(m.shape, dtype=np.uint8)
+        expect[idx[idx >= 0]] = 1
+        assert np.array_equal(m, expect), f"{name} unit {u} mask"
+        if akey == 0.0 and policy == 0:
+            assert per[I.ROLE_KEY] == 0
+
+
+def test_select_infeasible_budget_pads():
+    """More budget than eligible tokens: every eligible token is kept and the
+    tail of the row is -1."""
+    w = _w("llama8b", L=1, b=1, Hq=4, Hkv=1, n=600)
+    roles_np = np.full((1, 600), I.ROLE_KEY, dtype=np.uint8)
+    roles_np[0, ::10] = I.ROLE_VALUE
+    batch = lib_batch(w, DEV)
+    scores = _tied_scores(batch.score_shape(), 9)
+    keep = torch.empty(batch.kept_shape(0.5), dtype=torch.int32, device=DEV)
+    R.role_alloc_select(batch, scores, torch.as_tensor(roles_np, device=DEV),
+                        R.select_params(0.5, I.PAPER_ALPHA, 0.0, I.ROLE_KEY), keep)
+    torch.cuda.synchronize()
+    row = keep.cpu().numpy().reshape(-1)
+    assert row.size == 300
+    assert np.array_equal(row[:60], np.arange(0, 600, 10))
+    assert np.all(row[60:] == -1)
+
+
+# ----------------------------------------------------------------- compaction
+
+@pytest.mark.parametrize("varlen", [False, True])
+def test_kv_compact_bit_exact(varlen):
+    if varlen:
+        w = _w("ragged", L=2, b=3, Hq=8, Hkv=2, n=900, seqlens=(900, 0, 333))
+    else:
+        w = _w("llama8b", L=2, b=2, Hq=8, Hkv=2, n=1000)
+    B = 0.2
+    roles = I.workload_roles(w, 4)
+    K, V = I.make_kv(w, roles, 4, device=DEV)
+    batch = lib_batch(w, DEV)
+    rng = np.random.default_rng(11)
+    keep_np = np.full(batch.kept_shape(B), -1, dtype=np.int32)
+    ob = oracle_batch(w)
+    cu_kept = ob.kept_offsets(B)
+    for u in range(ob.n_units):
+        l, s, h = ob.unit(u)
+        n = ob.seqlens[s]
+        kcount = O.kept_count(n, B) if n else 0
+        take = max(0, kcount - 3)
+        idx = np.sort(rng.choice(n, size=take, replace=False)) if take else np.zeros(0, int)
+        row = np.full(kcount, -1, dtype=np.int32)
+        row[:take] = idx
+        if varlen:
+            keep_np[l, h, cu_kept[s]:cu_kept[s + 1]] = row
+        else:
+            keep_np.reshape(ob.n_units, -1)[u] = row
+    keep = torch.as_tensor(keep_np, device=DEV)
+    k_out = torch.full(R.compact_shape(batch, B), 3.0, dtype=torch.bfloat16, device=DEV)
+    v_out = torch.full_like(k_out, 3.0)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    R.kv_compact(batch, K, V, keep, B, k_out, v_out, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    kb, vb = I.bf16_bits(K), I.bf16_bits(V)
+    ko, vo = I.bf16_bits(k_out), I.bf16_bits(v_out)
+    for u in range(ob.n_units):
+        l, s, h = ob.unit(u)
+        if varlen:
+            sl = slice(cu_kept[s], cu_kept[s + 1])
+            row, kr, vr = keep_np[l, h, sl], ko[l, h, sl], vo[l, h, sl]
+        else:
+            row = keep_np.reshape(ob.n_units, -1)[u]
+            kr = ko.reshape(ob.n_units, -1, w.d)[u]
+            vr = vo.reshape(ob.n_units, -1, w.d)[u]
+        assert np.array_equal(kr, O.compact_unit(ob.kv_rows(kb, u), row))
+        assert np.array_equal(vr, O.compact_unit(ob.kv_rows(vb, u), row))
+        ok = row >= 0
+        ref_t = torch.index_select(torch.as_tensor(ob.kv_rows(kb, u).astype(np.int32)), 0,
+                                   torch.as_tensor(row[ok].astype(np.int64)))
+        assert np.array_equal(kr[ok].astype(np.int32), ref_t.numpy())
+
+
+# ------------------------------------------------------------- whole pipeline
+
+@pytest.mark.parametrize("name", ["tiny", "ragged_small"])
+def test_rolekv_compress_pipeline(name):
+    if name == "tiny":
+        w = I.WORKLOADS["tiny"]
+    else:
+        w = _w("ragged", L=2, b=4, Hq=14, Hkv=2, n=3000, seqlens=(3000, 1024, 77, 2222))
+    B = w.budgets[0]
+    roles_np, K, V, qw = _snapkv_inputs(w, seed=6)
+    batch = lib_batch(w, DEV)
+    params = R.select_params(B, I.PAPER_ALPHA, 0.0, I.ROLE_KEY)
+    keep = torch.empty(batch.kept_shape(B), dtype=torch.int32, device=DEV)
+    k_out = torch.empty(R.compact_shape(batch, B), dtype=torch.bfloat16, device=DEV)
+    v_out = torch.empty_like(k_out)
+    ws = R.workspace(R.OP_COMPRESS, batch, w.W)
+    roles = torch.as_tensor(roles_np, device=DEV)
+    R.rolekv_compress(batch, qw, K, V, w.W, w.pool_k, roles, params, keep, k_out, v_out, ws)
+    # the separate calls give the same kept set
+    scores = torch.empty(batch.score_shape(), dtype=torch.float32, device=DEV)
+    R.snapkv_score(batch, qw, K, w.W, w.pool_k, scores)
+    keep2 = torch.empty_like(keep)
+    R.role_alloc_select(batch, scores, roles, params, keep2)
+    torch.cuda.synchronize()
+    assert torch.equal(keep, keep2)
+    ob = oracle_batch(w)
+    ref = O.snapkv_batch(ob, I.bf16_bits(qw), I.bf16_bits(K), w.W, w.pool_k)
+    cu_kept = ob.kept_offsets(B)
+    keep_np = keep.cpu().numpy()
+    ko = I.bf16_bits(k_out)
+    kb = I.bf16_bits(K)
+    for u, (_, pooled) in ref.items():
+        l, s, h = ob.unit(u)
+        if ob.varlen:
+            row = keep_np[l, h, cu_kept[s]:cu_kept[s + 1]]
+            kr = ko[l, h, cu_kept[s]:cu_kept[s + 1]]
+        else:
+            row = keep_np.reshape(ob.n_units, -1)[u]
+            kr = ko.reshape(ob.n_units, -1, w.d)[u]
+        check_index_sets(ob, u, row, pooled, roles_np, I.N_ROLES, I.PAPER_ALPHA, I.ROLE_KEY, 0.0, B)
+        assert np.array_equal(kr, O.compact_unit(ob.kv_rows(kb, u), row))

@@ -1,0 +1,499 @@
+"""Benchmark of the role-conditional KV-eviction hot path on GB300.
+
+One step = the whole path over one batch of synthetic input: SnapKV windowed
+score (pass 1, normalisers, pass 2), the role-conditional selector with the
+max-pool fused into its load, and the K/V gather-compaction, for every
+(layer, sequence, KV head) of the workload.  The default workload is the
+long-context one the headline metric is quoted on: 32 layers, 4 sequences of
+32768 tokens, 32 query / 8 KV heads, head dim 128, W = 64, pool 7, B = 0.10
+(about 17 GB of bf16 K/V resident on the GPU, larger than L2, so no L2 flush
+is needed between steps).
+
+Prints one JSON line (rank 0).  `--impl reference` times the fp64 CPU oracle
+on a bounded sample of the same workload instead.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "KV tokens scored+compressed/sec at N=32k; % of GB300 HBM roofline"
+UNIT = "tokens/s"
+
+
+# ----------------------------------------------------------------- helpers --
+
+def dist_env():
+    return int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")), \
+        int(os.environ.get("LOCAL_RANK", "0"))
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    """Largest value of x over all ranks (x on every rank)."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained", d["bf16_tflops"]),
+                "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "source": "fallback"}
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(prefix="clocks_", suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        time.sleep(0.25)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for nm, v in zip(names, parts[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(nm)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------- algorithmic counts --
+
+def path_counts(w, B):
+    """Algorithmic bytes / flops per step of each kernel of the path (DESIGN
+    notes): K read once per pass, the window queries, the pre-pool score
+    written and read once, the kept K/V rows read and written, the kept index
+    written and read."""
+    U = w.L * w.b * w.Hkv
+    n = w.n
+    d = w.d
+    rows = w.G * w.W
+    K = math.ceil(B * n)
+    kbytes = U * n * d * 2
+    qbytes = U * rows * d * 2
+    flops = 2.0 * U * rows * n * d
+    return {
+        "pass1": {"bytes": kbytes + qbytes, "flops": flops},
+        "lse": {"bytes": U * rows * 4 * 3, "flops": 0.0},
+        "pass2": {"bytes": kbytes + qbytes + U * n * 4, "flops": flops},
+        "select": {"bytes": U * n * 4 + w.b * n + U * K * 4, "flops": 0.0},
+        "compact": {"bytes": U * K * 4 + 2 * 2 * U * K * d * 2, "flops": 0.0},
+        "path_bytes": kbytes + qbytes + U * n * 8 + U * K * 8 + 2 * 2 * U * K * d * 2 + w.b * n,
+        "kept": K,
+    }
+
+
+# ----------------------------------------------------------------- GPU arm --
+
+def run_gpu(args):
+    import torch
+
+    from paper_2607_13205_gb300 import inputs as I
+    from paper_2607_13205_gb300 import rolekv as R
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local)
+    w = I.WORKLOADS[args.workload]
+    if args.layers:
+        w = w.scaled(L=args.layers)
+    B = w.budgets[0]
+    if w.kind != "snapkv":
+        raise SystemExit("the bench times the SnapKV path")
+
+    roles_np = I.workload_roles(w, seed=rank)
+    K, V = I.make_kv(w, roles_np, seed=rank, device=dev)
+    qw = I.make_q_window(w, seed=rank, device=dev)
+    roles = torch.as_tensor(roles_np, device=dev)
+    batch = R.Batch(w.L, w.b, w.Hq, w.Hkv, w.d, w.n, seqlens=list(w.seqlens) if w.varlen else None,
+                    device=dev)
+    params = R.select_params(B, I.PAPER_ALPHA, alpha_key=0.0, key_role=I.ROLE_KEY)
+    scores = torch.empty(batch.score_shape(), dtype=torch.float32, device=dev)
+    keep = torch.empty(batch.kept_shape(B), dtype=torch.int32, device=dev)
+    k_out = torch.empty(R.compact_shape(batch, B), dtype=torch.bfloat16, device=dev)
+    v_out = torch.empty_like(k_out)
+    ws = R.workspace(R.OP_SNAPKV, batch, w.W, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    names = ["pass1", "lse", "pass2", "select", "compact"]
+
+    def step(ev=None):
+        # the path as three public calls: pre-pool scores (pool_k = 1 writes
+        # them straight out), selection with the pool fused, compaction
+        if ev is not None:
+            R.set_stage_events(ev[1:4])
+        R.snapkv_score(batch, qw, K, w.W, 1, scores, ws=ws, status=status, stream=stream)
+        if ev is not None:
+            R.set_stage_events(ev[4:5])
+        R.role_alloc_select(batch, scores, roles, params, keep, pool_k=w.pool_k, status=status,
+                            stream=stream)
+        if ev is not None:
+            R.set_stage_events(ev[5:6])
+        R.kv_compact(batch, K, V, keep, B, k_out, v_out, status=status, stream=stream)
+        if ev is not None:
+            R.set_stage_events([])
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize(dev)
+
+    # per-step events: [0] step start, [1..3] snapkv kernels, [4] select, [5] compact
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
+    for evs in events:
+        for e in evs:
+            e.record(stream)       # create the underlying CUDA events
+    torch.cuda.synchronize(dev)
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for i in range(args.steps):
+        events[i][0].record(stream)
+        step(events[i])
+    t1.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clock_info = clocks.stop()
+    elapsed_ms = t0.elapsed_time(t1)
+    elapsed_ms = max_over_ranks(elapsed_ms, world)
+    st = int(status.item())
+    if st != 0:
+        raise SystemExit(f"device status {st} during the timed steps")
+
+    per_kernel = {nm: 0.0 for nm in names}
+    for evs in events:
+        for j, nm in enumerate(names):
+            per_kernel[nm] += evs[j].elapsed_time(evs[j + 1])
+    per_kernel = {nm: v / args.steps for nm, v in per_kernel.items()}
+
+    seq_tokens = w.b * w.n if not w.varlen else sum(w.seqlens)
+    ms_step = elapsed_ms / args.steps
+    value = world * seq_tokens * args.steps / (elapsed_ms / 1e3)
+
+    peaks = load_peaks()
+    counts = path_counts(w, B)
+    dom = max(names, key=lambda k: per_kernel[k])
+    dk = counts[dom]
+    t_dom = per_kernel[dom] / 1e3
+    t_hbm = dk["bytes"] / (peaks["hbm_gbs"] * 1e9)
+    t_tc = dk["flops"] / (peaks["bf16_tflops"] * 1e12) if dk["flops"] else 0.0
+    if t_tc > t_hbm:
+        roof = {"bound": "tensor", "achieved": dk["flops"] / t_dom / 1e12,
+                "peak": peaks["bf16_tflops"], "unit": "TFLOP/s"}
+    else:
+        roof = {"bound": "hbm", "achieved": dk["bytes"] / t_dom / 1e9, "peak": peaks["hbm_gbs"],
+                "unit": "GB/s"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["kernel"] = dom
+    roof["traffic"] = args.traffic
+    roof["peak_source"] = peaks["source"] + " (burst)"
+    path_frac = counts["path_bytes"] / (ms_step / 1e3) / 1e9 / peaks["hbm_gbs"]
+
+    result = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"{w.name}: L={w.L} b={w.b} Hq={w.Hq} Hkv={w.Hkv} d={w.d} "
+                               f"N={w.n} W={w.W} pool={w.pool_k} B={B}",
+                   "global_batch": world * w.b, "seq_len": w.n, "parallelism": f"replicas x{world}",
+                   "l2": "inputs larger than L2 (17 GB K/V), no flush"},
+        "hbm_path_frac": path_frac,
+        "per_kernel_ms": per_kernel,
+        "unit_tokens_per_s": world * w.L * w.Hkv * seq_tokens * args.steps / (elapsed_ms / 1e3),
+        "roofline": roof,
+        "clocks": clock_info,
+        "gpu_launches": 5 * args.steps,
+    }
+
+    if not args.no_e2e:
+        result["e2e"] = run_e2e(args, w, B, batch, params, qw, K, V, roles, scores, keep, k_out,
+                                v_out, ws, status, stream, world, seq_tokens)
+    if rank == 0 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(w, B, args.cpu_seconds, host_inputs=(qw, K, V, roles_np))
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def run_e2e(args, w, B, batch, params, qw, K, V, roles, scores, keep, k_out, v_out, ws, status,
+            stream, world, seq_tokens):
+    """The same step through the public calls with host buffers: the step's
+    inputs are copied from pinned host memory and the kept indices and the
+    compressed K/V read back, inside the timed region."""
+    import torch
+
+    from paper_2607_13205_gb300 import rolekv as R
+
+    h_qw = torch.empty(qw.shape, dtype=qw.dtype, pin_memory=True)
+    h_k = torch.empty(K.shape, dtype=K.dtype, pin_memory=True)
+    h_v = torch.empty(V.shape, dtype=V.dtype, pin_memory=True)
+    h_roles = torch.empty(roles.shape, dtype=roles.dtype, pin_memory=True)
+    h_qw.copy_(qw)
+    h_k.copy_(K)
+    h_v.copy_(V)
+    h_roles.copy_(roles)
+    o_keep = torch.empty(keep.shape, dtype=keep.dtype, pin_memory=True)
+    o_k = torch.empty(k_out.shape, dtype=k_out.dtype, pin_memory=True)
+    o_v = torch.empty(v_out.shape, dtype=v_out.dtype, pin_memory=True)
+    torch.cuda.synchronize()
+    bi = sum(t.numel() * t.element_size() for t in (h_qw, h_k, h_v, h_roles))
+    bo = sum(t.numel() * t.element_size() for t in (o_keep, o_k, o_v))
+
+    def e2e_step():
+        qw.copy_(h_qw, non_blocking=True)
+        K.copy_(h_k, non_blocking=True)
+        V.copy_(h_v, non_blocking=True)
+        roles.copy_(h_roles, non_blocking=True)
+        R.snapkv_score(batch, qw, K, w.W, 1, scores, ws=ws, status=status, stream=stream)
+        R.role_alloc_select(batch, scores, roles, params, keep, pool_k=w.pool_k, status=status,
+                            stream=stream)
+        R.kv_compact(batch, K, V, keep, B, k_out, v_out, status=status, stream=stream)
+        o_keep.copy_(keep, non_blocking=True)
+        o_k.copy_(k_out, non_blocking=True)
+        o_v.copy_(v_out, non_blocking=True)
+
+    e2e_step()
+    torch.cuda.synchronize()
+    steps = max(1, min(args.steps, args.e2e_steps))
+    barrier(world)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        e2e_step()
+    torch.cuda.synchronize()
+    dt = time.perf_counter() - t0
+    barrier(world)
+    dt = max_over_ranks(dt, world)
+    return {"value": world * seq_tokens * steps / dt, "unit": UNIT, "h2d_bytes_per_step": bi,
+            "d2h_bytes_per_step": bo, "steps": steps, "ms_per_step": dt / steps * 1e3}
+
+
+# ------------------------------------------------------ CPU oracle baseline --
+
+def oracle_units(w, B, units, qw_bits, k_bits, v_bits, roles_np):
+    """Score, select and compact the given units with the fp64 oracle."""
+    from oracle import rolekv_oracle as O
+    from paper_2607_13205_gb300 import inputs as I
+
+    ob = O.Batch(w.L, w.b, w.Hq, w.Hkv, w.d, w.n, seqlens=list(w.seqlens) if w.varlen else None)
+    sc = O.snapkv_batch(ob, qw_bits, k_bits, w.W, w.pool_k, units=units)
+    sel = O.select_batch(ob, {u: sc[u][1] for u in sc}, roles_np, I.N_ROLES, I.PAPER_ALPHA,
+                         I.ROLE_KEY, 0.0, B)
+    for u, (idx, _) in sel.items():
+        O.compact_unit(ob.kv_rows(k_bits, u), idx)
+        O.compact_unit(ob.kv_rows(v_bits, u), idx)
+    return sel
+
+
+def _sample_arrays(w, units, host_inputs):
+    """Host bf16 bit arrays holding (at least) the sampled units' data."""
+    import numpy as np
+
+    from paper_2607_13205_gb300 import inputs as I
+
+    qw, K, V, roles_np = host_inputs
+    layers = sorted({u // (w.b * w.Hkv) for u in units})
+    assert layers == [0], "samples are taken from layer 0"
+    qb = np.zeros((w.L,) + tuple(qw.shape[1:]), dtype=np.uint16)
+    qb[0] = I.bf16_bits(qw[0])
+    kb = np.zeros((1,) + tuple(K.shape[1:]), dtype=np.uint16)
+    kb[0] = I.bf16_bits(K[0])
+    vb = np.zeros_like(kb)
+    vb[0] = I.bf16_bits(V[0])
+    return qb, kb, vb, roles_np
+
+
+def cpu_baseline(w, B, seconds: float, host_inputs):
+    """The oracle as it stands on this host's cores, on units of layer 0 of
+    the same workload until `seconds` of CPU work, extrapolated to a step."""
+    U = w.L * w.b * w.Hkv
+    per_layer = w.b * w.Hkv
+    units = []
+    qb = kb = vb = roles_np = None
+    t_total = 0.0
+    done = 0
+    while True:
+        u = done % per_layer
+        if qb is None:
+            qb, kb, vb, roles_np = _sample_arrays(w, [u], host_inputs)
+        t0 = time.perf_counter()
+        oracle_units(w, B, [u], qb, kb, vb, roles_np)
+        t_total += time.perf_counter() - t0
+        done += 1
+        units.append(u)
+        if t_total >= seconds or done >= per_layer:
+            break
+    seq_tokens = w.b * w.n if not w.varlen else sum(w.seqlens)
+    value = (done / U) * seq_tokens / t_total
+    return {"value": value, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
+            "sample": f"{done} of {U} (layer, sequence, KV head) units of layer 0, "
+                      f"{t_total:.1f} s, extrapolated linearly to the full step",
+            "seconds": t_total}
+
+
+def blas_threads() -> int:
+    for var in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
+        if os.environ.get(var):
+            try:
+                return int(os.environ[var])
+            except ValueError:
+                pass
+    return os.cpu_count() or 1
+
+
+def run_reference(args):
+    """The reference arm: the fp64 oracle, timed as it stands, each step a
+    bounded sample of the workload's units (rank 0 only)."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    import numpy as np
+    import torch
+
+    from paper_2607_13205_gb300 import inputs as I
+
+    w = I.WORKLOADS[args.workload]
+    B = w.budgets[0]
+    w1 = w.scaled(L=1)
+    roles_np = I.workload_roles(w1, seed=0)
+    K, V = I.make_kv(w1, roles_np, seed=0, device="cpu")
+    qw = I.make_q_window(w1, seed=0, device="cpu")
+    qb, kb, vb = I.bf16_bits(qw), I.bf16_bits(K), I.bf16_bits(V)
+    U = w.L * w.b * w.Hkv
+    per_step = max(1, args.ref_units)
+    seq_tokens = w.b * w.n
+    nxt = 0
+
+    def step():
+        nonlocal nxt
+        units = [(nxt + i) % (w1.b * w1.Hkv) for i in range(per_step)]
+        nxt += per_step
+        oracle_units(w1, B, units, qb, kb, vb, roles_np)
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    dt = time.perf_counter() - t0
+    value = (per_step * args.steps / U) * seq_tokens / dt
+    sample = (f"{per_step} of {U} (layer, sequence, KV head) units per step, extrapolated "
+              "linearly to the full workload")
+    out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": dt / args.steps * U / per_step * 1e3,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+           "data": "synthetic", "impl": "reference",
+           "config": {"workload": f"{w.name}: L={w.L} b={w.b} Hq={w.Hq} Hkv={w.Hkv} d={w.d} "
+                                  f"N={w.n} W={w.W} pool={w.pool_k} B={B}",
+                      "global_batch": w.b, "seq_len": w.n, "parallelism": "cpu"},
+           "cpu_baseline": {"value": value, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
+                            "sample": sample},
+           "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="long")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--ref-units", type=int, default=2)
+    ap.add_argument("--layers", type=int, default=0,
+                    help="override the layer count (smaller cases for profiling)")
+    ap.add_argument("--traffic", type=float, default=None,
+                    help="dram bytes per launch of the dominant kernel from an ncu capture")
+    args = ap.parse_args(argv)
+    if args.warmup < 3 and args.impl == "ours":
+        print("warning: fewer than 3 warm-up steps", file=sys.stderr)
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

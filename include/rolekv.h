@@ -154,6 +154,33 @@ int snapkv_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k
                  float* scores_prepool, void* workspace, size_t workspace_bytes,
                  int32_t* status_dev, void* stream);
 
+/* snapkv_score without a workspace (the paper has no counterpart; this is a
+ * deployment convenience of this library).  Some callers cannot allocate
+ * device memory at the point where they score: an inference server whose
+ * memory manager has already handed all of HBM to the KV cache and forbids
+ * further allocations, a plugin that is given only its input and output
+ * buffers, or a latency-critical path where cudaMalloc's device-wide
+ * synchronisation is not acceptable.  This call takes the same inputs and
+ * outputs as snapkv_score and keeps its scratch (the pass-1 partial row
+ * statistics and the per-row normalisers) in a static device array of
+ * 64 MiB that every GPU loading this library reserves until the process
+ * exits; it calls no cudaMalloc, cudaFree or other allocating routine.
+ *   Limits: batches whose scratch would exceed 64 MiB are rejected with
+ *   ROLEKV_ERR_UNSUPPORTED (about 9 MiB for 32 layers x 4 x 8 KV heads at
+ *   32768 tokens); with pool_k > 1, scores_prepool is required, because the
+ *   pre-pool scores are an output here, not scratch.
+ *   Set-up: the first call on each device looks up the array's device address
+ *   (cudaGetSymbolAddress) with that device current and caches it; make that
+ *   first call before any stream capture.
+ *   Sharing: every call on a device uses the same array and leaves its
+ *   contents behind; each call overwrites all it reads, so nothing needs
+ *   clearing, but calls that overlap on the GPU (other streams, other host
+ *   threads) race on the array -- order them on one stream. */
+int snapkv_score_noalloc(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k,
+                         int32_t W, int32_t pool_k, float scale, const float* lse_win,
+                         float* scores, float* scores_prepool, int32_t* status_dev,
+                         void* stream);
+
 /* H2O accumulated attention mass (Section 2): s(t) = sum over the G query heads
  * of the KV head and every causal query position q >= t of p_t(q).
  *   q       bf16 prefill queries of every position: dense [L][b][Hq][n][d] or

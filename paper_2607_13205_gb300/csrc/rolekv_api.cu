@@ -381,6 +381,44 @@ int fill_select(const BatchInfo& bi, const rolekv_batch* bt, const rolekv_select
 }  // namespace
 }  // namespace rolekv
 
+// ---------------------------------------------------- no-allocation variant --
+//
+// Scratch of snapkv_score_noalloc: the pass-1 partial row statistics and the
+// per-row normalisers, held in one file-scope device array so that callers who
+// cannot allocate device memory (see rolekv.h) still get the two-pass score.
+// Every GPU that loads this library reserves the array until the process exits.
+static constexpr size_t kNoAllocScratchBytes = size_t(64) << 20;
+static __device__ __align__(256) unsigned char rolekv_noalloc_scratch[kNoAllocScratchBytes];
+
+namespace rolekv {
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mutex;
+void* g_scratch_ptr[kMaxDevices] = {};
+
+// Device address of the scratch array on the current device.  The host-side
+// name of the array is only a stand-in, so the address is looked up once per
+// device, with that device current, and cached.
+int noalloc_scratch(void** out) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return fail(ROLEKV_ERR_UNSUPPORTED, "device %d out of range", dev);
+  std::lock_guard<std::mutex> lock(g_scratch_mutex);
+  if (g_scratch_ptr[dev] == nullptr) {
+    void* ptr = nullptr;
+    e = cudaGetSymbolAddress(&ptr, rolekv_noalloc_scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(scratch)");
+    g_scratch_ptr[dev] = ptr;
+  }
+  *out = g_scratch_ptr[dev];
+  return ROLEKV_OK;
+}
+
+}  // namespace
+}  // namespace rolekv
+
 using namespace rolekv;
 
 extern "C" {
@@ -571,6 +609,53 @@ int rolekv_compress(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tenso
                v_out, status_dev, &ca);
   e = launch_compact(ca, st);
   if (e != cudaSuccess) return cuda_fail(e, "kv_compact");
+  stage_mark(st);
+  return ROLEKV_OK;
+}
+
+int snapkv_score_noalloc(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k,
+                         int32_t W, int32_t pool_k, float scale, const float* lse_win,
+                         float* scores, float* scores_prepool, int32_t* status_dev,
+                         void* stream) {
+  BatchInfo bi;
+  int rc = check_batch(batch, &bi);
+  if (rc) return rc;
+  if (pool_k < 1 || pool_k > 15 || pool_k % 2 == 0)
+    return fail(ROLEKV_ERR_UNSUPPORTED, "pool_k=%d must be odd, 1..15", pool_k);
+  if (scores == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "scores is NULL");
+  if (pool_k > 1 && scores_prepool == nullptr)
+    return fail(ROLEKV_ERR_INVALID_ARG,
+                "snapkv_score_noalloc with pool_k > 1 needs scores_prepool (the pre-pool output)");
+  ScorePlan p;
+  rc = plan_score(kModeSnapKV, bi, W, lse_win == nullptr, false, &p);
+  if (rc) return rc;
+  if (p.bytes > kNoAllocScratchBytes)
+    return fail(ROLEKV_ERR_UNSUPPORTED,
+                "batch needs %zu bytes of scratch; snapkv_score_noalloc holds at most %zu "
+                "(use snapkv_score with a workspace)",
+                p.bytes, kNoAllocScratchBytes);
+  if ((rc = check_tensor("q_win", q_win, bi.d, bi.Hq, false, true))) return rc;
+  if ((rc = check_tensor("k", k, bi.d, bi.Hkv, bi.varlen, true))) return rc;
+  if (bi.n_max == 0) return ROLEKV_OK;
+  void* scratch = nullptr;
+  if ((rc = noalloc_scratch(&scratch))) return rc;
+  // Pass 1 writes every partial slot and the normaliser kernel every row
+  // before either is read, so nothing left by an earlier call is used.
+  if ((rc = bind_workspace(p, scratch, kNoAllocScratchBytes))) return rc;
+  float* pre = scores_prepool ? scores_prepool : scores;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  stage_begin();
+  rc = run_snapkv(bi, batch->cu_seqlens_dev, q_win, k, W, scale, lse_win, pre, p, status_dev, st);
+  if (rc) return rc;
+  if (pool_k == 1) {
+    if (pre == scores) return ROLEKV_OK;
+    cudaError_t e = cudaMemcpyAsync(scores, pre, static_cast<size_t>(score_elems(bi)) * 4,
+                                    cudaMemcpyDeviceToDevice, st);
+    if (e != cudaSuccess) return cuda_fail(e, "copy of pre-pool scores");
+    return ROLEKV_OK;
+  }
+  cudaError_t e = launch_maxpool(p.a, pre, scores, pool_k, st);
+  if (e != cudaSuccess) return cuda_fail(e, "max-pool");
   stage_mark(st);
   return ROLEKV_OK;
 }

@@ -60,6 +60,9 @@ _SIGNATURES = [
      [ctypes.POINTER(BatchDesc), Tensor, Tensor, ctypes.c_int32, ctypes.c_int32, ctypes.c_float,
       ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t,
       ctypes.c_void_p, ctypes.c_void_p]),
+    ("snapkv_score_noalloc", ctypes.c_int,
+     [ctypes.POINTER(BatchDesc), Tensor, Tensor, ctypes.c_int32, ctypes.c_int32, ctypes.c_float,
+      ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]),
     ("h2o_score", ctypes.c_int,
      [ctypes.POINTER(BatchDesc), Tensor, Tensor, ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p,
       ctypes.c_size_t, ctypes.c_void_p, ctypes.c_void_p]),
@@ -211,6 +214,19 @@ def snapkv_score(batch: Batch, q_win: torch.Tensor, k: torch.Tensor, W: int, poo
     _check(lib().snapkv_score(ctypes.byref(batch.desc), tensor_desc(q_win), tensor_desc(k, batch.varlen),
                               W, pool_k, scale, _ptr(lse_win), _ptr(scores), _ptr(scores_prepool),
                               _ptr(ws), ws.numel(), _ptr(status), _stream(stream)))
+    return scores
+
+
+def snapkv_score_noalloc(batch: Batch, q_win: torch.Tensor, k: torch.Tensor, W: int, pool_k: int,
+                         scores: torch.Tensor, scores_prepool: Optional[torch.Tensor] = None,
+                         lse_win: Optional[torch.Tensor] = None, scale: float = 0.0,
+                         status: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """snapkv_score for callers that cannot allocate device memory: no
+    workspace argument, the library's own static scratch is used instead
+    (see rolekv.h for its limit and sharing rules)."""
+    _check(lib().snapkv_score_noalloc(ctypes.byref(batch.desc), tensor_desc(q_win),
+                                      tensor_desc(k, batch.varlen), W, pool_k, scale, _ptr(lse_win),
+                                      _ptr(scores), _ptr(scores_prepool), _ptr(status), _stream(stream)))
     return scores
 
 

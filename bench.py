@@ -141,9 +141,8 @@ def path_counts(w, B):
     qbytes = U * rows * d * 2
     flops = 2.0 * U * rows * n * d
     return {
-        "pass1": {"bytes": kbytes + qbytes, "flops": flops},
-        "lse": {"bytes": U * rows * 4 * 3, "flops": 0.0},
-        "pass2": {"bytes": kbytes + qbytes + U * n * 4, "flops": flops},
+        # both passes in one kernel: K crosses HBM once, the QK^T is done twice
+        "score": {"bytes": kbytes + qbytes + U * n * 4, "flops": 2 * flops},
         "select": {"bytes": U * n * 4 + w.b * n + U * K * 4, "flops": 0.0},
         "compact": {"bytes": U * K * 4 + 2 * 2 * U * K * d * 2, "flops": 0.0},
         "path_bytes": kbytes + qbytes + U * n * 8 + U * K * 8 + 2 * 2 * U * K * d * 2 + w.b * n,
@@ -187,20 +186,20 @@ def run_gpu(args):
     status = torch.zeros(1, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream(dev)
 
-    names = ["pass1", "lse", "pass2", "select", "compact"]
+    names = ["score", "select", "compact"]
 
     def step(ev=None):
         # the path as three public calls: pre-pool scores (pool_k = 1 writes
         # them straight out), selection with the pool fused, compaction
         if ev is not None:
-            R.set_stage_events(ev[1:4])
+            R.set_stage_events(ev[1:2])
         R.snapkv_score(batch, qw, K, w.W, 1, scores, ws=ws, status=status, stream=stream)
         if ev is not None:
-            R.set_stage_events(ev[4:5])
+            R.set_stage_events(ev[2:3])
         R.role_alloc_select(batch, scores, roles, params, keep, pool_k=w.pool_k, status=status,
                             stream=stream)
         if ev is not None:
-            R.set_stage_events(ev[5:6])
+            R.set_stage_events(ev[3:4])
         R.kv_compact(batch, K, V, keep, B, k_out, v_out, status=status, stream=stream)
         if ev is not None:
             R.set_stage_events([])
@@ -209,8 +208,8 @@ def run_gpu(args):
         step()
     torch.cuda.synchronize(dev)
 
-    # per-step events: [0] step start, [1..3] snapkv kernels, [4] select, [5] compact
-    events = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
+    # per-step events: [0] step start, [1] score kernel, [2] select, [3] compact
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
     for evs in events:
         for e in evs:
             e.record(stream)       # create the underlying CUDA events
@@ -278,7 +277,7 @@ def run_gpu(args):
         "unit_tokens_per_s": world * w.L * w.Hkv * seq_tokens * args.steps / (elapsed_ms / 1e3),
         "roofline": roof,
         "clocks": clock_info,
-        "gpu_launches": 5 * args.steps,
+        "gpu_launches": 3 * args.steps,
     }
 
     if not args.no_e2e:

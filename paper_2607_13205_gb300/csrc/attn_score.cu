@@ -16,7 +16,7 @@
 // In both passes one producer warp streams 128-key K tiles and 256-row query
 // blocks into 128-byte-swizzled shared memory with TMA, one warp issues
 // tcgen05.mma (bf16 operands, fp32 accumulators in tensor memory, two
-// accumulator buffers) and eight epilogue warps drain the accumulators with
+// accumulator buffers) and sixteen epilogue warps drain the accumulators with
 // tcgen05.ld.  Every wait is an mbarrier wait bounded in time.
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -31,9 +31,10 @@ namespace rolekv {
 namespace {
 
 constexpr int kTileKeys = 128;
-constexpr int kEpiWarps = 8;
-constexpr int kProducerWarp = 8;
-constexpr int kMmaWarp = 9;
+constexpr int kEpiWarps = 16;                 // four per SM sub-partition
+constexpr int kParts = kEpiWarps / 4;         // epilogue warps sharing a TMEM lane quadrant
+constexpr int kProducerWarp = kEpiWarps;
+constexpr int kMmaWarp = kEpiWarps + 1;
 constexpr int kThreads = (kEpiWarps + 2) * 32;
 constexpr int kRowsMax = 256;
 constexpr uint32_t kTmemCols = 512;
@@ -56,8 +57,8 @@ struct Cfg {
   static constexpr int kLseOff = kKOff + SK * kKTileBytes;
   static constexpr int kPosOff = kLseOff + SQ * kRowsMax * 4;
   static constexpr int kRedOff = kPosOff + SQ * kRowsMax * 4;
-  static constexpr int kMergeOff = kRedOff + kTileKeys * 4;
-  static constexpr int kBarOff = kMergeOff + kRowsMax * 8;
+  static constexpr int kMergeOff = kRedOff + (kParts - 1) * kTileKeys * 4;
+  static constexpr int kBarOff = kMergeOff + kParts * kRowsMax * 8;
   static constexpr int kNumBars = 2 * SK + 2 * SQ + 4 + 3;
   static constexpr int kMiscOff = kBarOff + kNumBars * 8;
   static constexpr int kBytes = kMiscOff + 16;
@@ -239,6 +240,262 @@ __device__ __forceinline__ int64_t score_base(const ScoreArgs& a, const Unit& un
   return static_cast<int64_t>(u) * a.n_max;
 }
 
+// ---------------------------------------------------------------- epilogue --
+
+// NCOL accumulator columns of the calling thread's TMEM lane, as raw bits.
+// One wait for all loads; the fence keeps their uses below the wait.
+template <int NCOL>
+__device__ __forceinline__ void tmem_load_cols(uint32_t taddr, uint32_t* r) {
+  __syncwarp();
+#pragma unroll
+  for (int c = 0; c < NCOL / 32; ++c) tmem_ld32(taddr + c * 32, r + c * 32);
+  tmem_wait_ld();
+#pragma unroll
+  for (int c = 0; c < NCOL / 32; ++c) tmem_reg_fence(r + c * 32);
+}
+
+__device__ __forceinline__ float2 bits2(const uint32_t* r, int i) {
+  return make_float2(__uint_as_float(r[i]), __uint_as_float(r[i + 1]));
+}
+
+__device__ __forceinline__ float2 exp2x2(float2 v) {
+  return make_float2(fast_exp2(v.x), fast_exp2(v.y));
+}
+
+// sum_i exp2(v_i * c - m): packed f32x2 FMA/ADD, four independent partial sums.
+template <int NCOL>
+__device__ __forceinline__ float sum_exp2_shift(const uint32_t* r, float c, float m) {
+  const float2 cc = make_float2(c, c), mm = make_float2(-m, -m);
+  float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                   make_float2(0.f, 0.f)};
+#pragma unroll
+  for (int i = 0; i < NCOL; i += 8) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      acc[k] = __fadd2_rn(acc[k], exp2x2(__ffma2_rn(bits2(r, i + 2 * k), cc, mm)));
+  }
+  const float2 s = __fadd2_rn(__fadd2_rn(acc[0], acc[1]), __fadd2_rn(acc[2], acc[3]));
+  return s.x + s.y;
+}
+
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+template <int NCOL>
+__device__ __forceinline__ float max_cols(const uint32_t* r) {
+  float m[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) m[k] = __uint_as_float(r[k]);
+#pragma unroll
+  for (int i = 4; i + 8 <= NCOL; i += 8)
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      m[k] = max3f(m[k], __uint_as_float(r[i + 2 * k]), __uint_as_float(r[i + 2 * k + 1]));
+  // the last 4 columns
+#pragma unroll
+  for (int k = 0; k < 4; ++k) m[k] = fmaxf(m[k], __uint_as_float(r[NCOL - 4 + k]));
+  return fmaxf(fmaxf(m[0], m[1]), fmaxf(m[2], m[3]));
+}
+
+// One tile of pass 1 for the row at position `pos`: keys t0 .. t0+NCOL-1 with
+// raw logits r.  (m2, l) is the running reference and sum of exp2 relative
+// to it.  When the tile is fully visible and a reference exists, the tile is
+// summed against the current reference; a sum that is non-finite or above
+// 1e18 (a much larger logit arrived) is redone with the tile's exact max.
+template <int NCOL>
+__device__ __forceinline__ void rowstats_tile(const uint32_t* r, int t0, int pos, float c1,
+                                              float& m2, float& l) {
+  if (pos < 0 || t0 > pos) return;
+  const bool whole = (t0 + NCOL - 1 <= pos);
+  if (whole && m2 > -INFINITY) {
+    const float s = sum_exp2_shift<NCOL>(r, c1, m2);
+    if (s <= 1.0e18f) {
+      l += s;
+      return;
+    }
+  }
+  float mx, s;
+  if (whole) {
+    mx = max_cols<NCOL>(r) * c1;
+    const float mnew = fmaxf(m2, mx);
+    s = sum_exp2_shift<NCOL>(r, c1, mnew);
+    l = l * fast_exp2(m2 - mnew) + s;
+    m2 = mnew;
+  } else {
+    mx = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < NCOL; ++i)
+      if (t0 + i <= pos) mx = fmaxf(mx, __uint_as_float(r[i]));
+    const float mnew = fmaxf(m2, mx * c1);
+    s = 0.f;
+#pragma unroll
+    for (int i = 0; i < NCOL; ++i) {
+      const float e = fast_exp2(fmaf(__uint_as_float(r[i]), c1, -mnew));
+      s += (t0 + i <= pos) ? e : 0.f;
+    }
+    l = l * fast_exp2(m2 - mnew) + s;
+    m2 = mnew;
+  }
+}
+
+// Pass 1 epilogue: the thread owns one query row and NCOL keys of every tile.
+// With two row tiles, two parts share each tile (NCOL = 64 keys each); with
+// one, all four parts share it (NCOL = 32).  The parts merge at the end.
+template <int NCOL>
+__device__ __forceinline__ void rowstats_epilogue(const ScoreArgs& a, const Work& w, Shared& sh,
+                                                  uint32_t tmem, int n, int warp, int lane,
+                                                  int nrt) {
+  const int qd = warp & 3;
+  const int part = warp >> 2;
+  const int rt = (nrt == 2) ? part >> 1 : 0;
+  const int sub = (nrt == 2) ? part & 1 : part;
+  const int row = rt * 128 + qd * 32 + lane;
+  const int col0 = rt * 128 + sub * NCOL;
+  const int key0 = sub * NCOL;
+  const uint32_t lane_base = static_cast<uint32_t>(qd * 32) << 16;
+  const int rb = w.rb0;
+  const int pos = (w.rb1 > w.rb0) ? row_position(a, n, rb, row) : -1;
+  float m2 = -INFINITY, l = 0.f;
+  bool ok = true;
+  int pair = 0;
+  for (int kt = w.kt0; kt < w.kt1; ++kt) {
+    const int ab = pair & 1;
+    ok = __all_sync(0xffffffffu, mbar_wait(&sh.acc_full[ab], (pair >> 1) & 1, sh.abort_flag, a.status));
+    if (!ok) break;
+    tc_fence_after();
+    // 32 columns at a time keeps the live registers within the launch bound;
+    // the accumulator is released once its last columns are in registers.
+    uint32_t r[32];
+#pragma unroll
+    for (int h = 0; h < NCOL / 32; ++h) {
+      tmem_load_cols<32>(tmem + lane_base + ab * 256 + col0 + h * 32, r);
+      if (h + 1 == NCOL / 32) {
+        tc_fence_before();
+        mbar_arrive(&sh.acc_empty[ab]);
+      }
+      rowstats_tile<32>(r, kt * kTileKeys + key0 + h * 32, pos, a.c1, m2, l);
+    }
+    ++pair;
+  }
+  if (!ok) return;
+  const int nsub = kParts / nrt;            // parts sharing one row
+  if (sub != 0) {
+    sh.merge[sub * kRowsMax + row] = make_float2(m2, l);
+    mbar_arrive(sh.red_full);
+    return;
+  }
+  if (!mbar_wait(sh.red_full, 0, sh.abort_flag, a.status)) return;
+  for (int x = 1; x < nsub; ++x) {
+    const float2 o = sh.merge[x * kRowsMax + row];
+    const float mm = fmaxf(m2, o.x);
+    if (mm > -INFINITY) {
+      l = l * fast_exp2(m2 - mm) + o.y * fast_exp2(o.x - mm);
+      m2 = mm;
+    }
+  }
+  if (a.mode == kModeSnapKV) {
+    const int64_t slot = static_cast<int64_t>(w.u) * a.n_chunks + w.chunk;
+    a.partials[slot * kRowsMax + row] = make_float2(m2, l);
+    if (nrt == 1) a.partials[slot * kRowsMax + 128 + row] = make_float2(-INFINITY, 0.f);
+  } else if (w.rb1 > w.rb0) {
+    const int64_t o = (static_cast<int64_t>(w.u) * a.nrb_max + rb) * kRowsMax;
+    a.lse2[o + row] = (l > 0.f) ? m2 + __log2f(l) : INFINITY;
+    if (nrt == 1) a.lse2[o + 128 + row] = INFINITY;
+  }
+}
+
+// Pass 2 epilogue: the thread owns key lane `kl` of the tile and NCOL query
+// rows (one quarter of the block); the parts add up at the end of each tile.
+// sh.lse holds the negated log2 normalisers (-inf for rows that do not exist).
+template <int SQ, int NCOL>
+__device__ __forceinline__ void colsum_epilogue(const ScoreArgs& a, const Work& w, Shared& sh,
+                                                uint32_t tmem, int n, int warp, int lane,
+                                                bool q_streams) {
+  const int qd = warp & 3;
+  const int part = warp >> 2;
+  const uint32_t lane_base = static_cast<uint32_t>(qd * 32) << 16;
+  const int kl = qd * 32 + lane;
+  const int j0 = part * NCOL;
+  const int64_t sbase = score_base(a, w.unit, w.u);
+  const float c1 = a.c1;
+  const float2 cc = make_float2(c1, c1);
+  bool ok = true;
+  int pair = 0, quse = 0, xchg = 0;
+  for (int kt = w.kt0; kt < w.kt1 && ok; ++kt) {
+    const int t = kt * kTileKeys + kl;
+    float colsum = 0.f;
+    for (int rb = w.rb0; rb < w.rb1; ++rb) {
+      if (q_streams || kt == w.kt0) {
+        // Acquire the producer's normalisers and positions for this block.
+        ok = __all_sync(0xffffffffu, mbar_wait(&sh.q_full[quse % SQ], (quse / SQ) & 1,
+                                               sh.abort_flag, a.status));
+        if (!ok) break;
+        ++quse;
+      }
+      const int qslot = (quse - 1) % SQ;
+      int min_pos;
+      bool all_rows;
+      row_block_span(a, n, rb, &min_pos, &all_rows);
+      const bool fast = all_rows && (kt * kTileKeys + kTileKeys - 1 <= min_pos);
+      const int ab = pair & 1;
+      ok = __all_sync(0xffffffffu, mbar_wait(&sh.acc_full[ab], (pair >> 1) & 1, sh.abort_flag, a.status));
+      if (!ok) break;
+      tc_fence_after();
+      uint32_t r[NCOL];
+      tmem_load_cols<NCOL>(tmem + lane_base + ab * 256 + j0, r);
+      tc_fence_before();
+      mbar_arrive(&sh.acc_empty[ab]);
+      const float* nl = sh.lse + qslot * kRowsMax + j0;
+      if (fast) {
+        float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                         make_float2(0.f, 0.f)};
+#pragma unroll
+        for (int i = 0; i < NCOL; i += 8) {
+          const float4 L0 = *reinterpret_cast<const float4*>(nl + i);
+          const float4 L1 = *reinterpret_cast<const float4*>(nl + i + 4);
+          acc[0] = __fadd2_rn(acc[0], exp2x2(__ffma2_rn(bits2(r, i), cc, make_float2(L0.x, L0.y))));
+          acc[1] = __fadd2_rn(acc[1], exp2x2(__ffma2_rn(bits2(r, i + 2), cc, make_float2(L0.z, L0.w))));
+          acc[2] = __fadd2_rn(acc[2], exp2x2(__ffma2_rn(bits2(r, i + 4), cc, make_float2(L1.x, L1.y))));
+          acc[3] = __fadd2_rn(acc[3], exp2x2(__ffma2_rn(bits2(r, i + 6), cc, make_float2(L1.z, L1.w))));
+        }
+        const float2 s2 = __fadd2_rn(__fadd2_rn(acc[0], acc[1]), __fadd2_rn(acc[2], acc[3]));
+        colsum += s2.x + s2.y;
+      } else {
+        const int32_t* pos = sh.pos + qslot * kRowsMax + j0;
+        float s = 0.f;
+#pragma unroll
+        for (int i = 0; i < NCOL; ++i) {
+          const float e = fast_exp2(fmaf(__uint_as_float(r[i]), c1, nl[i]));
+          s += (t <= pos[i]) ? e : 0.f;
+        }
+        colsum += s;
+      }
+      if (q_streams || kt + 1 == w.kt1) mbar_arrive(&sh.q_empty[qslot]);
+      ++pair;
+    }
+    if (!ok) break;
+    // Add the row parts of this key and write s(t).
+    if (part != 0) {
+      ok = mbar_wait(sh.red_empty, (xchg & 1) ^ 1, sh.abort_flag, a.status);
+      if (!ok) break;
+      sh.red[(part - 1) * kTileKeys + kl] = colsum;
+      mbar_arrive(sh.red_full);
+    } else {
+      ok = mbar_wait(sh.red_full, xchg & 1, sh.abort_flag, a.status);
+      if (!ok) break;
+      float total = colsum;
+#pragma unroll
+      for (int x = 1; x < kParts; ++x) total += sh.red[(x - 1) * kTileKeys + kl];
+      mbar_arrive(sh.red_empty);
+      if (t < n) a.prepool[sbase + t] = total;
+    }
+    ++xchg;
+  }
+}
+
 // ------------------------------------------------------------------ kernel --
 
 template <int D, int PASS>
@@ -272,7 +529,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&sh.acc_full[i], 1);
       mbar_init(&sh.acc_empty[i], kEpiWarps * 32);
     }
-    mbar_init(sh.red_full, 128);
+    // non-leader parts hand their partial results to the leader part
+    mbar_init(sh.red_full, PASS == kPassColsum ? (kParts - 1) * 128 : (kParts - nrt) * 128);
     mbar_init(sh.red_empty, 128);
     mbar_init(sh.drain, 1);
     *sh.abort_flag = 0;
@@ -338,7 +596,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int j = lane; j < kRowsMax; j += 32) {
             const int p = row_position(a, n, rb, j);
             sh.pos[slot * kRowsMax + j] = p;
-            sh.lse[slot * kRowsMax + j] = (p >= 0) ? a.lse2[lrow + j] : INFINITY;
+            sh.lse[slot * kRowsMax + j] = (p >= 0) ? -a.lse2[lrow + j] : -INFINITY;
           }
         }
         if (lane == 0) {
@@ -442,159 +700,481 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else {
     // ------------------------------------------------------------- epilogue
-    const int qd = warp & 3;
-    const int hf = warp >> 2;
-    const uint32_t lane_base = static_cast<uint32_t>(qd * 32) << 16;
-    const float c1 = a.c1;
-    int pair = 0;
-    bool ok = true;
     if (PASS == kPassRowstats) {
-      // The thread owns query row `row`.  With two row tiles each half of the
-      // epilogue takes one tile; with one, the halves split the key columns
-      // of every tile and merge at the end.
-      const int row = (nrt == 2) ? hf * 128 + qd * 32 + lane : qd * 32 + lane;
-      const int col0 = (nrt == 2) ? hf * 128 : hf * 64;
-      const int key0 = (nrt == 2) ? 0 : hf * 64;
-      const int nchunk = (nrt == 2) ? 4 : 2;
-      const int rb = w.rb0;
-      const int pos = (w.rb1 > w.rb0) ? row_position(a, n, rb, row) : -1;
+      if (nrt == 2)
+        rowstats_epilogue<64>(a, w, sh, tmem, n, warp, lane, nrt);
+      else
+        rowstats_epilogue<32>(a, w, sh, tmem, n, warp, lane, nrt);
+    } else {
+      if (a.nrows_pad == 256)
+        colsum_epilogue<C::SQ, 64>(a, w, sh, tmem, n, warp, lane, q_streams);
+      else
+        colsum_epilogue<C::SQ, 32>(a, w, sh, tmem, n, warp, lane, q_streams);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ------------------------------------------------------------ fused SnapKV --
+
+template <int D>
+struct FCfg {
+  static constexpr int kHalves = D / 64;
+  static constexpr int kKSteps = D / 16;
+  static constexpr int kKTileBytes = kTileKeys * D * 2;
+  static constexpr int kQSlotBytes = kRowsMax * D * 2;
+  static constexpr int kKHalfBytes = kTileKeys * 128;
+  static constexpr int kQHalfBytes = kRowsMax * 128;
+  static constexpr int SK = 4;
+  static constexpr int kQOff = 0;
+  static constexpr int kKOff = kQOff + kQSlotBytes;
+  static constexpr int kLseOff = kKOff + SK * kKTileBytes;
+  static constexpr int kPosOff = kLseOff + kRowsMax * 4;
+  static constexpr int kRedOff = kPosOff + kRowsMax * 4;
+  static constexpr int kMergeOff = kRedOff + (kParts - 1) * kTileKeys * 4;
+  static constexpr int kBarOff = kMergeOff + kParts * kRowsMax * 8;
+  // k_full/k_empty[SK], q_full, q_empty, acc_full[2], acc_empty[2], merge_full,
+  // red_full, red_empty, drain, pub, lse_go, lse_ready
+  static constexpr int kNumBars = 2 * SK + 13;
+  static constexpr int kMiscOff = kBarOff + kNumBars * 8;
+  static constexpr int kBytes = kMiscOff + 32;
+  static constexpr int kSmemAlloc = kBytes + 1024;
+};
+
+struct FShared {
+  uint8_t* q;
+  uint8_t* k;
+  float* lse;        // negated log2 normalisers of the current item's rows
+  int32_t* pos;
+  float* red;
+  float2* merge;
+  uint64_t *k_full, *k_empty, *q_full, *q_empty, *acc_full, *acc_empty;
+  uint64_t *merge_full, *red_full, *red_empty, *drain;
+  uint64_t *pub, *lse_go, *lse_ready;
+  uint32_t* tmem_base;
+  volatile int* abort_flag;
+};
+
+template <int D>
+__device__ __forceinline__ FShared fcarve(uint8_t* raw) {
+  using C = FCfg<D>;
+  const uint32_t a = smem_u32(raw);
+  uint8_t* base = raw + ((1024u - (a & 1023u)) & 1023u);
+  FShared s;
+  s.q = base + C::kQOff;
+  s.k = base + C::kKOff;
+  s.lse = reinterpret_cast<float*>(base + C::kLseOff);
+  s.pos = reinterpret_cast<int32_t*>(base + C::kPosOff);
+  s.red = reinterpret_cast<float*>(base + C::kRedOff);
+  s.merge = reinterpret_cast<float2*>(base + C::kMergeOff);
+  uint64_t* b = reinterpret_cast<uint64_t*>(base + C::kBarOff);
+  s.k_full = b;
+  s.k_empty = b + C::SK;
+  b += 2 * C::SK;
+  s.q_full = b++;
+  s.q_empty = b++;
+  s.acc_full = b;
+  b += 2;
+  s.acc_empty = b;
+  b += 2;
+  s.merge_full = b++;
+  s.red_full = b++;
+  s.red_empty = b++;
+  s.drain = b++;
+  s.pub = b++;
+  s.lse_go = b++;
+  s.lse_ready = b++;
+  s.tmem_base = reinterpret_cast<uint32_t*>(base + C::kMiscOff);
+  s.abort_flag = reinterpret_cast<volatile int*>(base + C::kMiscOff + 4);
+  return s;
+}
+
+__device__ __forceinline__ int ld_acquire_gpu(const int32_t* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Key-tile range of chunk c of a unit with n keys.
+__device__ __forceinline__ void chunk_tiles(const ScoreArgs& a, int n, int c, int* kt0, int* kt1) {
+  const int ntiles = (n + kTileKeys - 1) / kTileKeys;
+  *kt0 = c * a.chunk_tiles;
+  *kt1 = min(ntiles, *kt0 + a.chunk_tiles);
+  if (*kt1 < *kt0) *kt1 = *kt0;
+}
+
+template <int D>
+__device__ __forceinline__ void issue_mma_rows_on_lanes(uint32_t qbase, uint32_t kbase,
+                                                        uint32_t dcol, int nrt) {
+  using C = FCfg<D>;
+  const uint32_t idesc = idesc_bf16_f32(128, kTileKeys);
+  for (int rt = 0; rt < nrt; ++rt) {
+#pragma unroll
+    for (int ks = 0; ks < C::kKSteps; ++ks) {
+      const uint32_t koff = (ks & 3) * 32;
+      const uint64_t ad =
+          sdesc_kmajor_sw128(qbase + (ks >> 2) * C::kQHalfBytes + rt * 128 * 128 + koff);
+      const uint64_t bd = sdesc_kmajor_sw128(kbase + (ks >> 2) * C::kKHalfBytes + koff);
+      mma_bf16_ss(dcol + rt * kTileKeys, ad, bd, idesc, ks > 0 ? 1u : 0u);
+    }
+  }
+}
+
+template <int D>
+__device__ __forceinline__ void issue_mma_keys_on_lanes(uint32_t qbase, uint32_t kbase,
+                                                        uint32_t dcol, int nrows_pad) {
+  using C = FCfg<D>;
+  const uint32_t idesc = idesc_bf16_f32(128, nrows_pad);
+#pragma unroll
+  for (int ks = 0; ks < C::kKSteps; ++ks) {
+    const uint32_t koff = (ks & 3) * 32;
+    const uint64_t ad = sdesc_kmajor_sw128(kbase + (ks >> 2) * C::kKHalfBytes + koff);
+    const uint64_t bd = sdesc_kmajor_sw128(qbase + (ks >> 2) * C::kQHalfBytes + koff);
+    mma_bf16_ss(dcol, ad, bd, idesc, ks > 0 ? 1u : 0u);
+  }
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    snapkv_fused_kernel(const __grid_constant__ CUtensorMap k_map,
+                        const __grid_constant__ CUtensorMap q_map, const FusedArgs fa) {
+  using C = FCfg<D>;
+  const ScoreArgs& a = fa.s;
+  extern __shared__ uint8_t smem_raw[];
+  FShared sh = fcarve<D>(smem_raw);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int nrt = a.nrows_pad / 128;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < C::SK; ++i) {
+      mbar_init(&sh.k_full[i], 1);
+      mbar_init(&sh.k_empty[i], 1);
+    }
+    mbar_init(sh.q_full, 1);
+    mbar_init(sh.q_empty, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&sh.acc_full[i], 1);
+      mbar_init(&sh.acc_empty[i], kEpiWarps * 32);
+    }
+    mbar_init(sh.merge_full, (kParts - nrt) * 128);
+    mbar_init(sh.red_full, (kParts - 1) * 128);
+    mbar_init(sh.red_empty, 128);
+    mbar_init(sh.drain, 1);
+    mbar_init(sh.pub, kEpiWarps * 32);
+    mbar_init(sh.lse_go, 1);
+    mbar_init(sh.lse_ready, kEpiWarps * 32);
+    *sh.abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (a.nrows < a.nrows_pad) {
+    const int words = (a.nrows_pad - a.nrows) * 32;
+    for (int hf = 0; hf < C::kHalves; ++hf) {
+      uint32_t* dst = reinterpret_cast<uint32_t*>(sh.q + hf * C::kQHalfBytes + a.nrows * 128);
+      for (int i = threadIdx.x; i < words; i += kThreads) dst[i] = 0u;
+    }
+    fence_proxy_async_smem();
+  }
+  if (warp == kMmaWarp) {
+    tmem_alloc(sh.tmem_base, kTmemCols);
+    tmem_relinquish();
+  }
+  if (warp == kProducerWarp && lane == 0) {
+    tma_prefetch_map(&k_map);
+    tma_prefetch_map(&q_map);
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *sh.tmem_base;
+
+  if (warp == kProducerWarp) {
+    // ------------------------------------------------------------- producer
+    if (lane == 0) {
+      // Pass-1 tiles and the window queries are read again soon (pass 2, the
+      // unit's other chunks): keep them in L2; pass-2 reads are their last.
+      const uint64_t keep = l2_policy_evict_last();
+      const uint64_t drop = l2_policy_evict_first();
+      int kload = 0, qload = 0;
+      // Items are dealt round-robin: the grid is a multiple of the chunks per
+      // unit, so a unit's chunks run on different CTAs in the same round.
+      for (int item = blockIdx.x; item < fa.n_items; item += gridDim.x) {
+        const Unit un = decode_unit(a, item / a.n_chunks);
+        int kt0, kt1;
+        chunk_tiles(a, un.n, item % a.n_chunks, &kt0, &kt1);
+        if (kt1 == kt0) continue;
+        // window queries of the unit
+        if (!mbar_wait(sh.q_empty, (qload & 1) ^ 1, sh.abort_flag, a.status)) break;
+        mbar_arrive_expect_tx(sh.q_full, static_cast<uint32_t>(a.nrows) * D * 2);
+        for (int g = 0; g < a.G; ++g) {
+          const Coord c = tma_coord(a.q_layer, a.q_seq, a.q_head, a.q_tok, false, un,
+                                    un.h * a.G + g, 0);
+#pragma unroll
+          for (int hf = 0; hf < C::kHalves; ++hf)
+            tma_load_2d_hint(sh.q + hf * C::kQHalfBytes + g * a.P * 128, &q_map, c.x + hf * 64,
+                             c.y, sh.q_full, keep);
+        }
+        ++qload;
+        // the chunk's key tiles, once for each pass
+        bool ok = true;
+        for (int pass = 0; pass < 2 && ok; ++pass)
+          for (int kt = kt0; kt < kt1; ++kt) {
+            const int slot = kload % C::SK;
+            if (!mbar_wait(&sh.k_empty[slot], ((kload / C::SK) & 1) ^ 1, sh.abort_flag, a.status)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&sh.k_full[slot], C::kKTileBytes);
+            const Coord c = tma_coord(a.k_layer, a.k_seq, a.k_head, a.k_tok, a.varlen != 0, un,
+                                      un.h, static_cast<int64_t>(kt) * kTileKeys);
+#pragma unroll
+            for (int hf = 0; hf < C::kHalves; ++hf)
+              tma_load_2d_hint(sh.k + slot * C::kKTileBytes + hf * C::kKHalfBytes, &k_map,
+                               c.x + hf * 64, c.y, &sh.k_full[slot], pass == 0 ? keep : drop);
+            ++kload;
+          }
+        if (!ok) break;
+      }
+      if (*sh.abort_flag) {
+        for (int i = 0; i < min(kload, C::SK); ++i) {
+          const int ld = kload - 1 - i;
+          mbar_wait(&sh.k_full[ld % C::SK], (ld / C::SK) & 1, nullptr, nullptr);
+        }
+        if (qload > 0) mbar_wait(sh.q_full, (qload - 1) & 1, nullptr, nullptr);
+      }
+    }
+    __syncwarp();
+  } else if (warp == kMmaWarp) {
+    // ------------------------------------------------------------------ MMA
+    if (lane == 0) {
+      int kuse = 0, quse = 0, pair = 0;
+      bool ok = true;
+      for (int item = blockIdx.x; item < fa.n_items && ok; item += gridDim.x) {
+        const Unit un = decode_unit(a, item / a.n_chunks);
+        int kt0, kt1;
+        chunk_tiles(a, un.n, item % a.n_chunks, &kt0, &kt1);
+        if (kt1 == kt0) continue;
+        if (!mbar_wait(sh.q_full, quse & 1, sh.abort_flag, a.status)) break;
+        ++quse;
+        const uint32_t qbase = smem_u32(sh.q);
+        for (int pass = 0; pass < 2 && ok; ++pass)
+          for (int kt = kt0; kt < kt1; ++kt) {
+            const int kslot = kuse % C::SK;
+            const int ab = pair & 1;
+            if (!mbar_wait(&sh.k_full[kslot], (kuse / C::SK) & 1, sh.abort_flag, a.status) ||
+                !mbar_wait(&sh.acc_empty[ab], ((pair >> 1) & 1) ^ 1, sh.abort_flag, a.status)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t kbase = smem_u32(sh.k + kslot * C::kKTileBytes);
+            if (pass == 0)
+              issue_mma_rows_on_lanes<D>(qbase, kbase, tmem + ab * 256, nrt);
+            else
+              issue_mma_keys_on_lanes<D>(qbase, kbase, tmem + ab * 256, a.nrows_pad);
+            mma_commit(&sh.acc_full[ab]);
+            mma_commit(&sh.k_empty[kslot]);
+            ++kuse;
+            ++pair;
+          }
+        if (ok) mma_commit(sh.q_empty);
+      }
+      mma_commit(sh.drain);
+      mbar_wait(sh.drain, 0, nullptr, nullptr);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------- epilogue
+    const int qd = warp & 3;
+    const int part = warp >> 2;
+    const uint32_t lane_base = static_cast<uint32_t>(qd * 32) << 16;
+    const int etid = threadIdx.x;                  // 0 .. kEpiWarps*32-1
+    // pass 1 mapping: one query row, a slice of every tile's keys
+    const int rt = (nrt == 2) ? part >> 1 : 0;
+    const int sub = (nrt == 2) ? part & 1 : part;
+    const int row = rt * 128 + qd * 32 + lane;
+    const int p1cols = (nrt == 2) ? 64 : 32;
+    const int col1 = rt * 128 + sub * p1cols;
+    const int nsub = kParts / nrt;
+    // pass 2 mapping: one key lane, a quarter of the rows
+    const int kl = qd * 32 + lane;
+    const int p2cols = a.nrows_pad / kParts;
+    const int j0 = part * p2cols;
+    const float c1 = a.c1;
+    const float2 cc = make_float2(c1, c1);
+    int pair = 0, xchg = 0;
+    bool ok = true;
+    int ipop = 0;                                  // items done: barrier phases
+    for (int item = blockIdx.x; item < fa.n_items && ok; item += gridDim.x, ++ipop) {
+      const int u = item / a.n_chunks;
+      const int chunk = item % a.n_chunks;
+      const Unit un = decode_unit(a, u);
+      const int n = un.n;
+      int kt0, kt1;
+      chunk_tiles(a, n, chunk, &kt0, &kt1);
+
+      // ---- pass 1: running (max2, sum) of this thread's row over its keys
+      const int pos = row_position(a, n, 0, row);
       float m2 = -INFINITY, l = 0.f;
-      for (int kt = w.kt0; kt < w.kt1 && ok; ++kt) {
+      for (int kt = kt0; kt < kt1; ++kt) {
         const int ab = pair & 1;
         ok = __all_sync(0xffffffffu, mbar_wait(&sh.acc_full[ab], (pair >> 1) & 1, sh.abort_flag, a.status));
         if (!ok) break;
         tc_fence_after();
-        for (int c = 0; c < nchunk; ++c) {
-          uint32_t r[32];
-          __syncwarp();
-          tmem_ld32(tmem + lane_base + ab * 256 + col0 + c * 32, r);
-          tmem_wait_ld();
-          tmem_reg_fence(r);
-          const int t0 = kt * kTileKeys + key0 + c * 32;
-          if (pos >= 0 && t0 <= pos) {
-            const bool whole = (t0 + 31 <= pos);
-            float mx = -INFINITY;
-#pragma unroll
-            for (int i = 0; i < 32; ++i)
-              if (whole || t0 + i <= pos) mx = fmaxf(mx, __uint_as_float(r[i]));
-            const float mnew = fmaxf(m2, mx * c1);
-            float acc = 0.f;
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const float e = fast_exp2(fmaf(__uint_as_float(r[i]), c1, -mnew));
-              acc += (whole || t0 + i <= pos) ? e : 0.f;
-            }
-            l = l * fast_exp2(m2 - mnew) + acc;
-            m2 = mnew;
+        uint32_t r[32];
+        for (int h = 0; h < p1cols / 32; ++h) {
+          tmem_load_cols<32>(tmem + lane_base + ab * 256 + col1 + h * 32, r);
+          if (h + 1 == p1cols / 32) {
+            tc_fence_before();
+            mbar_arrive(&sh.acc_empty[ab]);
           }
+          rowstats_tile<32>(r, kt * kTileKeys + sub * p1cols + h * 32, pos, c1, m2, l);
         }
-        tc_fence_before();
-        mbar_arrive(&sh.acc_empty[ab]);
         ++pair;
       }
-      bool writer = (nrt == 2) || (hf == 0);
-      if (nrt == 1 && ok) {
-        // Merge the two column halves of each row.
-        if (hf == 1) {
-          sh.merge[row] = make_float2(m2, l);
-          mbar_arrive(sh.red_full);
-        } else {
-          ok = mbar_wait(sh.red_full, 0, sh.abort_flag, a.status);
-          if (ok) {
-            const float2 o = sh.merge[row];
-            const float mm = fmaxf(m2, o.x);
-            if (mm > -INFINITY) {
-              l = l * fast_exp2(m2 - mm) + o.y * fast_exp2(o.x - mm);
-              m2 = mm;
-            }
+      if (!ok) break;
+      // merge the key slices of each row, publish the chunk's partials
+      if (sub != 0) {
+        sh.merge[sub * kRowsMax + row] = make_float2(m2, l);
+        mbar_arrive(sh.merge_full);
+      } else {
+        ok = mbar_wait(sh.merge_full, ipop & 1, sh.abort_flag, a.status);
+        for (int x = 1; x < nsub && ok; ++x) {
+          const float2 o = sh.merge[x * kRowsMax + row];
+          const float mm = fmaxf(m2, o.x);
+          if (mm > -INFINITY) {
+            l = l * fast_exp2(m2 - mm) + o.y * fast_exp2(o.x - mm);
+            m2 = mm;
           }
         }
+        const int64_t slot = static_cast<int64_t>(u) * a.n_chunks + chunk;
+        a.partials[slot * kRowsMax + row] = make_float2(m2, l);
+        if (nrt == 1) a.partials[slot * kRowsMax + 128 + row] = make_float2(-INFINITY, 0.f);
+        __threadfence();
       }
-      writer = writer && ok;
-      if (writer) {
-        if (a.mode == kModeSnapKV) {
-          const int64_t slot = static_cast<int64_t>(w.u) * a.n_chunks + w.chunk;
-          a.partials[slot * kRowsMax + row] = make_float2(m2, l);
-          if (nrt == 1) a.partials[slot * kRowsMax + 128 + row] = make_float2(-INFINITY, 0.f);
-        } else if (w.rb1 > w.rb0) {
-          const int64_t o = (static_cast<int64_t>(w.u) * a.nrb_max + rb) * kRowsMax;
-          a.lse2[o + row] = (l > 0.f) ? m2 + __log2f(l) : INFINITY;
-          if (nrt == 1) a.lse2[o + 128 + row] = INFINITY;
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) break;
+      mbar_arrive(sh.pub);
+      if (etid == 0) {
+        // every row of this chunk is visible: count it, then wait for the
+        // unit's other chunks (bounded)
+        bool got = mbar_wait(sh.pub, ipop & 1, sh.abort_flag, a.status);
+        if (got) {
+          __threadfence();
+          atomicAdd(fa.work + 1 + u, 1);
+          const uint64_t t0 = global_timer_ns();
+          while (ld_acquire_gpu(fa.work + 1 + u) < a.n_chunks) {
+            if (*sh.abort_flag || global_timer_ns() - t0 > kWaitLimitNs) {
+              *sh.abort_flag = 1;
+              if (a.status) atomicOr(a.status, ROLEKV_STATUS_TIMEOUT);
+              got = false;
+              break;
+            }
+            __nanosleep(128);
+          }
         }
+        mbar_arrive(sh.lse_go);
       }
-    } else {
-      // The thread owns key lane `kl` of the tile; the two halves split the
-      // query rows and add up at the end of each key tile.
-      const int kl = qd * 32 + lane;
-      const int half_cols = a.nrows_pad / 2;
-      const int nchunk = half_cols / 32;
-      const int j0 = hf * half_cols;
-      const int64_t sbase = score_base(a, w.unit, w.u);
-      int quse = 0, xchg = 0;
-      for (int kt = w.kt0; kt < w.kt1 && ok; ++kt) {
+      ok = __all_sync(0xffffffffu, mbar_wait(sh.lse_go, ipop & 1, sh.abort_flag, a.status));
+      if (!ok || *sh.abort_flag) break;
+      // ---- normalisers of the unit's rows from all chunks' partials
+      if (etid < kRowsMax) {
+        const int j = etid;
+        const int p = row_position(a, n, 0, j);
+        float nl = -INFINITY;
+        if (p >= 0) {
+          // one online merge over the chunks, eight independent loads in flight
+          const float2* part_j = a.partials + static_cast<int64_t>(u) * a.n_chunks * kRowsMax + j;
+          float m = -INFINITY, s = 0.f;
+          for (int c0 = 0; c0 < a.n_chunks; c0 += 8) {
+            float2 v[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+              v[i] = (c0 + i < a.n_chunks) ? __ldcg(&part_j[(c0 + i) * kRowsMax])
+                                           : make_float2(-INFINITY, 0.f);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              if (v[i].y > 0.f) {
+                const float mn = fmaxf(m, v[i].x);
+                s = s * exp2f(m - mn) + v[i].y * exp2f(v[i].x - mn);
+                m = mn;
+              }
+            }
+          }
+          if (s > 0.f) nl = -(m + log2f(s));
+        }
+        sh.lse[j] = nl;
+        sh.pos[j] = p;
+      }
+      mbar_arrive(sh.lse_ready);
+      ok = __all_sync(0xffffffffu, mbar_wait(sh.lse_ready, ipop & 1, sh.abort_flag, a.status));
+      if (!ok) break;
+
+      // ---- pass 2: column sums of this thread's key over its rows
+      int min_pos;
+      bool all_rows;
+      row_block_span(a, n, 0, &min_pos, &all_rows);
+      const int64_t sbase = score_base(a, un, u);
+      for (int kt = kt0; kt < kt1; ++kt) {
         const int t = kt * kTileKeys + kl;
-        float colsum = 0.f;
-        for (int rb = w.rb0; rb < w.rb1; ++rb) {
-          const bool new_q = q_streams || kt == w.kt0;
-          if (new_q) {
-            // Acquire the producer's normalisers and positions for this block.
-            ok = __all_sync(0xffffffffu, mbar_wait(&sh.q_full[quse % C::SQ], (quse / C::SQ) & 1,
-                                                   sh.abort_flag, a.status));
-            if (!ok) break;
-            ++quse;
-          }
-          const int qslot = (quse - 1) % C::SQ;
-          int min_pos;
-          bool all_rows;
-          row_block_span(a, n, rb, &min_pos, &all_rows);
-          const bool fast = all_rows && (kt * kTileKeys + kTileKeys - 1 <= min_pos);
-          const int ab = pair & 1;
-          ok = __all_sync(0xffffffffu, mbar_wait(&sh.acc_full[ab], (pair >> 1) & 1, sh.abort_flag, a.status));
-          if (!ok) break;
-          tc_fence_after();
-          const float* lse = sh.lse + qslot * kRowsMax + j0;
-          const int32_t* pos = sh.pos + qslot * kRowsMax + j0;
-          for (int c = 0; c < nchunk; ++c) {
-            uint32_t r[32];
-            __syncwarp();
-            tmem_ld32(tmem + lane_base + ab * 256 + j0 + c * 32, r);
-            tmem_wait_ld();
-            tmem_reg_fence(r);
-            float acc = 0.f;
-            if (fast) {
-#pragma unroll
-              for (int i = 0; i < 32; i += 4) {
-                const float4 L4 = *reinterpret_cast<const float4*>(lse + c * 32 + i);
-                acc += fast_exp2(fmaf(__uint_as_float(r[i + 0]), c1, -L4.x));
-                acc += fast_exp2(fmaf(__uint_as_float(r[i + 1]), c1, -L4.y));
-                acc += fast_exp2(fmaf(__uint_as_float(r[i + 2]), c1, -L4.z));
-                acc += fast_exp2(fmaf(__uint_as_float(r[i + 3]), c1, -L4.w));
-              }
-            } else {
-#pragma unroll
-              for (int i = 0; i < 32; ++i) {
-                const float e = fast_exp2(fmaf(__uint_as_float(r[i]), c1, -lse[c * 32 + i]));
-                acc += (t <= pos[c * 32 + i]) ? e : 0.f;
-              }
-            }
-            colsum += acc;
-          }
-          tc_fence_before();
-          mbar_arrive(&sh.acc_empty[ab]);
-          if (q_streams || kt + 1 == w.kt1) mbar_arrive(&sh.q_empty[qslot]);
-          ++pair;
-        }
+        const bool fast = all_rows && (kt * kTileKeys + kTileKeys - 1 <= min_pos);
+        const int ab = pair & 1;
+        ok = __all_sync(0xffffffffu, mbar_wait(&sh.acc_full[ab], (pair >> 1) & 1, sh.abort_flag, a.status));
         if (!ok) break;
-        // Add the two row halves of this key and write s(t).
-        if (hf == 1) {
+        tc_fence_after();
+        float colsum = 0.f;
+        uint32_t r[32];
+        for (int h = 0; h < p2cols / 32; ++h) {
+          tmem_load_cols<32>(tmem + lane_base + ab * 256 + j0 + h * 32, r);
+          if (h + 1 == p2cols / 32) {
+            tc_fence_before();
+            mbar_arrive(&sh.acc_empty[ab]);
+          }
+          const float* nlp = sh.lse + j0 + h * 32;
+          if (fast) {
+            float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                             make_float2(0.f, 0.f)};
+#pragma unroll
+            for (int i = 0; i < 32; i += 8) {
+              const float4 L0 = *reinterpret_cast<const float4*>(nlp + i);
+              const float4 L1 = *reinterpret_cast<const float4*>(nlp + i + 4);
+              acc[0] = __fadd2_rn(acc[0], exp2x2(__ffma2_rn(bits2(r, i), cc, make_float2(L0.x, L0.y))));
+              acc[1] = __fadd2_rn(acc[1], exp2x2(__ffma2_rn(bits2(r, i + 2), cc, make_float2(L0.z, L0.w))));
+              acc[2] = __fadd2_rn(acc[2], exp2x2(__ffma2_rn(bits2(r, i + 4), cc, make_float2(L1.x, L1.y))));
+              acc[3] = __fadd2_rn(acc[3], exp2x2(__ffma2_rn(bits2(r, i + 6), cc, make_float2(L1.z, L1.w))));
+            }
+            const float2 s2 = __fadd2_rn(__fadd2_rn(acc[0], acc[1]), __fadd2_rn(acc[2], acc[3]));
+            colsum += s2.x + s2.y;
+          } else {
+            const int32_t* pp = sh.pos + j0 + h * 32;
+            float s = 0.f;
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const float e = fast_exp2(fmaf(__uint_as_float(r[i]), c1, nlp[i]));
+              s += (t <= pp[i]) ? e : 0.f;
+            }
+            colsum += s;
+          }
+        }
+        ++pair;
+        // add the row parts of this key and write s(t)
+        if (part != 0) {
           ok = mbar_wait(sh.red_empty, (xchg & 1) ^ 1, sh.abort_flag, a.status);
           if (!ok) break;
-          sh.red[kl] = colsum;
+          sh.red[(part - 1) * kTileKeys + kl] = colsum;
           mbar_arrive(sh.red_full);
         } else {
           ok = mbar_wait(sh.red_full, xchg & 1, sh.abort_flag, a.status);
           if (!ok) break;
-          const float total = colsum + sh.red[kl];
+          float total = colsum;
+#pragma unroll
+          for (int x = 1; x < kParts; ++x) total += sh.red[(x - 1) * kTileKeys + kl];
           mbar_arrive(sh.red_empty);
           if (t < n) a.prepool[sbase + t] = total;
         }
@@ -685,6 +1265,47 @@ cudaError_t launch_attn_pass(int pass, int d, const CUtensorMap& kmap, const CUt
                      : launch_pass<128, kPassColsum>(kmap, qmap, a, grid, stream);
   return pass == 0 ? launch_pass<64, kPassRowstats>(kmap, qmap, a, grid, stream)
                    : launch_pass<64, kPassColsum>(kmap, qmap, a, grid, stream);
+}
+
+template <int D>
+static cudaError_t launch_fused(const CUtensorMap& kmap, const CUtensorMap& qmap,
+                                const FusedArgs& a, cudaStream_t stream) {
+  using C = FCfg<D>;
+  cudaError_t e = cudaFuncSetAttribute(snapkv_fused_kernel<D>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemAlloc);
+  if (e != cudaSuccess) return e;
+  int dev = 0, sms = 0, per_sm = 0;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+  if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, snapkv_fused_kernel<D>, kThreads,
+                                                         C::kSmemAlloc)) != cudaSuccess)
+    return e;
+  if (per_sm < 1) return cudaErrorInvalidConfiguration;
+  // One CTA per SM, all resident at once (the per-unit arrival counters are
+  // waited on), which the cooperative launch guarantees.  The grid is a
+  // multiple of the chunks per unit so that items dealt round-robin put all
+  // of a unit's chunks in the same round.
+  const int nc = a.s.n_chunks;
+  if (nc < 1 || nc > sms) return cudaErrorInvalidConfiguration;
+  const int grid = (sms / nc) * nc;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(grid));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = C::kSmemAlloc;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, snapkv_fused_kernel<D>, kmap, qmap, a);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
+cudaError_t launch_snapkv_fused(int d, const CUtensorMap& kmap, const CUtensorMap& qmap,
+                                const FusedArgs& a, cudaStream_t stream) {
+  return d == 128 ? launch_fused<128>(kmap, qmap, a, stream) : launch_fused<64>(kmap, qmap, a, stream);
 }
 
 cudaError_t launch_snapkv_lse(const ScoreArgs& a, const float* lse_win, cudaStream_t stream) {

@@ -38,6 +38,20 @@ struct ScoreArgs {
 
 cudaError_t launch_attn_pass(int pass, int d, const CUtensorMap& kmap, const CUtensorMap& qmap,
                              const ScoreArgs& a, int grid, cudaStream_t stream);
+
+// The SnapKV score in one persistent, cooperative launch: (unit, chunk of
+// key tiles) items are dealt round-robin to the CTAs; each runs pass 1 on its
+// chunk, meets the unit's other chunks at a bounded arrival counter, forms
+// the exact normalisers from their partials and runs pass 2 on the same (now
+// L2-resident) tiles.
+struct FusedArgs {
+  ScoreArgs s;                      // s.n_chunks = chunks per unit, s.chunk_tiles = tiles per chunk
+  int32_t* work;                    // [1 + u]: chunks of unit u done with pass 1 ([0] unused)
+  int32_t n_items;
+};
+
+cudaError_t launch_snapkv_fused(int d, const CUtensorMap& kmap, const CUtensorMap& qmap,
+                                const FusedArgs& a, cudaStream_t stream);
 cudaError_t launch_snapkv_lse(const ScoreArgs& a, const float* lse_win, cudaStream_t stream);
 cudaError_t launch_maxpool(const ScoreArgs& a, const float* in, float* out, int pool_k,
                            cudaStream_t stream);

@@ -173,18 +173,29 @@ int num_sms() {
 
 struct ScorePlan {
   ScoreArgs a;
-  size_t off_partials, off_lse, off_prepool, bytes;
+  size_t off_partials, off_lse, off_prepool, off_work, bytes;
   int grid1, grid2;
+  bool fused;
+  int32_t n_items;
+  int32_t* work;
 };
+
+// Key tiles per work item of the fused SnapKV kernel: small enough that a
+// chunk's tiles are still in L2 when pass 2 reads them again, large enough to
+// amortise the per-unit meeting point.  Eight chunks per unit at most: the
+// grid (152 SMs = 19 x 8) deals a unit's chunks to CTAs of the same round.
+constexpr int kFusedChunkTiles = 32;
+constexpr int kFusedMaxChunks = 8;
 
 int64_t score_elems(const BatchInfo& bi) {
   return bi.varlen ? static_cast<int64_t>(bi.L) * bi.Hkv * bi.T : bi.n_units * bi.n_max;
 }
 
 int plan_score(int mode, const BatchInfo& bi, int W, bool need_partials, bool need_prepool,
-               ScorePlan* p) {
+               ScorePlan* p, bool fused = false) {
   ScoreArgs& a = p->a;
   std::memset(&a, 0, sizeof(a));
+  p->fused = fused && mode == kModeSnapKV;
   if (bi.d != 64 && bi.d != 128)
     return fail(ROLEKV_ERR_UNSUPPORTED, "head dim %d (the score kernels take 64 or 128)", bi.d);
   a.L = bi.L;
@@ -210,11 +221,20 @@ int plan_score(int mode, const BatchInfo& bi, int W, bool need_partials, bool ne
   a.nrows_pad = a.nrows <= 128 ? 128 : 256;
   const int ntiles = (bi.n_max + kTileKeys - 1) / kTileKeys;
   if (mode == kModeSnapKV) {
-    a.chunk_tiles = ntiles < 64 ? (ntiles > 0 ? ntiles : 1) : 64;
+    if (p->fused) {
+      // at most kFusedMaxChunks chunks per unit (they must all be resident at
+      // once), of about kFusedChunkTiles tiles when the sequence allows
+      int nc = (ntiles + kFusedChunkTiles - 1) / kFusedChunkTiles;
+      nc = nc < 1 ? 1 : (nc > kFusedMaxChunks ? kFusedMaxChunks : nc);
+      a.chunk_tiles = ntiles > 0 ? (ntiles + nc - 1) / nc : 1;
+    } else {
+      a.chunk_tiles = ntiles < 64 ? (ntiles > 0 ? ntiles : 1) : 64;
+    }
     a.n_chunks = (ntiles + a.chunk_tiles - 1) / a.chunk_tiles;
     if (a.n_chunks < 1) a.n_chunks = 1;
     p->grid1 = a.n_units * a.n_chunks;
     p->grid2 = p->grid1;
+    p->n_items = a.n_units * a.n_chunks;
     a.nrb_max = 1;
   } else {
     a.nrb_max = (bi.n_max + a.P - 1) / a.P;
@@ -228,6 +248,8 @@ int plan_score(int mode, const BatchInfo& bi, int W, bool need_partials, bool ne
   off += align256(static_cast<size_t>(a.n_units) * a.nrb_max * kRowsMax * 4);
   p->off_prepool = off;
   if (need_prepool) off += align256(static_cast<size_t>(score_elems(bi)) * 4);
+  p->off_work = off;
+  if (p->fused) off += align256((static_cast<size_t>(a.n_units) + 1) * 4);
   p->bytes = off;
   return ROLEKV_OK;
 }
@@ -251,6 +273,7 @@ int bind_workspace(ScorePlan& p, void* ws, size_t ws_bytes) {
   uint8_t* base = static_cast<uint8_t*>(ws);
   p.a.partials = reinterpret_cast<float2*>(base + p.off_partials);
   p.a.lse2 = reinterpret_cast<float*>(base + p.off_lse);
+  p.work = p.fused ? reinterpret_cast<int32_t*>(base + p.off_work) : nullptr;
   return ROLEKV_OK;
 }
 
@@ -273,6 +296,19 @@ int run_snapkv(const BatchInfo& bi, const int32_t* cu_seqlens, const rolekv_tens
   rc = make_row_map(&qmap, q_win, tensor_span(q_win, bi.L, bi.b, bi.Hq, W, bi.d, false), W);
   if (rc) return rc;
   cudaError_t e;
+  if (lse_win == nullptr && p.fused) {
+    // one persistent launch: both passes, normalisers formed in-kernel
+    FusedArgs fa;
+    fa.s = a;
+    fa.work = p.work;
+    fa.n_items = p.n_items;
+    e = cudaMemsetAsync(p.work, 0, (static_cast<size_t>(a.n_units) + 1) * 4, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "clearing the work counters");
+    e = launch_snapkv_fused(bi.d, kmap, qmap, fa, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "snapkv fused score");
+    stage_mark(stream);
+    return ROLEKV_OK;
+  }
   if (lse_win == nullptr) {
     e = launch_attn_pass(0, bi.d, kmap, qmap, a, p.grid1, stream);
     if (e != cudaSuccess) return cuda_fail(e, "snapkv pass 1");
@@ -439,9 +475,9 @@ int rolekv_workspace_size(int op, const rolekv_batch* batch, int32_t W, size_t* 
   if (rc) return rc;
   ScorePlan p;
   switch (op) {
-    case 0: rc = plan_score(kModeSnapKV, bi, W, true, true, &p); break;
+    case 0: rc = plan_score(kModeSnapKV, bi, W, true, true, &p, true); break;
     case 1: rc = plan_score(kModeH2O, bi, 0, false, false, &p); break;
-    case 2: rc = plan_score(kModeSnapKV, bi, W, true, true, &p); break;
+    case 2: rc = plan_score(kModeSnapKV, bi, W, true, true, &p, true); break;
     default: return fail(ROLEKV_ERR_INVALID_ARG, "unknown op %d", op);
   }
   if (rc) return rc;
@@ -460,7 +496,7 @@ int snapkv_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k
     return fail(ROLEKV_ERR_UNSUPPORTED, "pool_k=%d must be odd, 1..15", pool_k);
   if (scores == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "scores is NULL");
   ScorePlan p;
-  rc = plan_score(kModeSnapKV, bi, W, lse_win == nullptr, scores_prepool == nullptr, &p);
+  rc = plan_score(kModeSnapKV, bi, W, lse_win == nullptr, scores_prepool == nullptr, &p, true);
   if (rc) return rc;
   if ((rc = check_tensor("q_win", q_win, bi.d, bi.Hq, false, true))) return rc;
   if ((rc = check_tensor("k", k, bi.d, bi.Hkv, bi.varlen, true))) return rc;
@@ -579,7 +615,7 @@ int rolekv_compress(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tenso
   if (pool_k < 1 || pool_k > 15 || pool_k % 2 == 0)
     return fail(ROLEKV_ERR_UNSUPPORTED, "pool_k=%d must be odd, 1..15", pool_k);
   ScorePlan p;
-  rc = plan_score(kModeSnapKV, bi, W, true, true, &p);
+  rc = plan_score(kModeSnapKV, bi, W, true, true, &p, true);
   if (rc) return rc;
   SelectArgs sa;
   if ((rc = fill_select(bi, batch, params, &sa))) return rc;

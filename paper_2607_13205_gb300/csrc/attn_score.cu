@@ -740,8 +740,8 @@ struct FCfg {
   static constexpr int kMergeOff = kRedOff + (kParts - 1) * kTileKeys * 4;
   static constexpr int kBarOff = kMergeOff + kParts * kRowsMax * 8;
   // k_full/k_empty[SK], q_full, q_empty, acc_full[2], acc_empty[2], merge_full,
-  // red_full, red_empty, drain, pub, lse_go, lse_ready
-  static constexpr int kNumBars = 2 * SK + 13;
+  // red_full[2], red_empty[2], drain, pub, lse_go, lse_ready
+  static constexpr int kNumBars = 2 * SK + 15;
   static constexpr int kMiscOff = kBarOff + kNumBars * 8;
   static constexpr int kBytes = kMiscOff + 32;
   static constexpr int kSmemAlloc = kBytes + 1024;
@@ -784,8 +784,10 @@ __device__ __forceinline__ FShared fcarve(uint8_t* raw) {
   s.acc_empty = b;
   b += 2;
   s.merge_full = b++;
-  s.red_full = b++;
-  s.red_empty = b++;
+  s.red_full = b;
+  b += 2;
+  s.red_empty = b;
+  b += 2;
   s.drain = b++;
   s.pub = b++;
   s.lse_go = b++;
@@ -861,11 +863,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(sh.q_empty, 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(&sh.acc_full[i], 1);
-      mbar_init(&sh.acc_empty[i], kEpiWarps * 32);
+      mbar_init(&sh.acc_empty[i], (kEpiWarps / 2) * 32);   // one group per buffer
+      mbar_init(&sh.red_full[i], 128);
+      mbar_init(&sh.red_empty[i], 128);
     }
     mbar_init(sh.merge_full, (kParts - nrt) * 128);
-    mbar_init(sh.red_full, (kParts - 1) * 128);
-    mbar_init(sh.red_empty, 128);
     mbar_init(sh.drain, 1);
     mbar_init(sh.pub, kEpiWarps * 32);
     mbar_init(sh.lse_go, 1);
@@ -991,21 +993,29 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else {
     // ------------------------------------------------------------- epilogue
-    const int qd = warp & 3;
-    const int part = warp >> 2;
+    // Two groups of eight warps own the two accumulator buffers (group g the
+    // tiles with pair parity g): while one group computes on its tile the
+    // other drains the next one from tensor memory.
+    const int grp = warp >> 3;
+    const int gw = warp & 7;
+    const int qd = gw & 3;
+    const int gp = gw >> 2;                        // part within the group
     const uint32_t lane_base = static_cast<uint32_t>(qd * 32) << 16;
     const int etid = threadIdx.x;                  // 0 .. kEpiWarps*32-1
-    // pass 1 mapping: one query row, a slice of every tile's keys
-    const int rt = (nrt == 2) ? part >> 1 : 0;
-    const int sub = (nrt == 2) ? part & 1 : part;
+    // pass 1 mapping: one query row and all keys of each owned tile (two row
+    // tiles) or half of them (one row tile); the row's partial sums from the
+    // other group / part merge at the end of the chunk
+    const int rt = (nrt == 2) ? gp : 0;
+    const int sub = (nrt == 2) ? grp : grp * 2 + gp;
     const int row = rt * 128 + qd * 32 + lane;
-    const int p1cols = (nrt == 2) ? 64 : 32;
-    const int col1 = rt * 128 + sub * p1cols;
+    const int p1cols = (nrt == 2) ? 128 : 64;
+    const int col1 = rt * 128 + ((nrt == 2) ? 0 : gp * 64);
+    const int key1 = (nrt == 2) ? 0 : gp * 64;
     const int nsub = kParts / nrt;
-    // pass 2 mapping: one key lane, a quarter of the rows
+    // pass 2 mapping: one key lane, half of the rows of each owned tile
     const int kl = qd * 32 + lane;
-    const int p2cols = a.nrows_pad / kParts;
-    const int j0 = part * p2cols;
+    const int p2cols = a.nrows_pad / 2;
+    const int j0 = gp * p2cols;
     const float c1 = a.c1;
     const float2 cc = make_float2(c1, c1);
     int pair = 0, xchg = 0;
@@ -1022,8 +1032,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       // ---- pass 1: running (max2, sum) of this thread's row over its keys
       const int pos = row_position(a, n, 0, row);
       float m2 = -INFINITY, l = 0.f;
-      for (int kt = kt0; kt < kt1; ++kt) {
+      for (int kt = kt0; kt < kt1; ++kt, ++pair) {
         const int ab = pair & 1;
+        if (ab != grp) continue;                   // the other group's tile
         ok = __all_sync(0xffffffffu, mbar_wait(&sh.acc_full[ab], (pair >> 1) & 1, sh.abort_flag, a.status));
         if (!ok) break;
         tc_fence_after();
@@ -1034,9 +1045,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_before();
             mbar_arrive(&sh.acc_empty[ab]);
           }
-          rowstats_tile<32>(r, kt * kTileKeys + sub * p1cols + h * 32, pos, c1, m2, l);
+          rowstats_tile<32>(r, kt * kTileKeys + key1 + h * 32, pos, c1, m2, l);
         }
-        ++pair;
       }
       if (!ok) break;
       // merge the key slices of each row, publish the chunk's partials
@@ -1121,10 +1131,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool all_rows;
       row_block_span(a, n, 0, &min_pos, &all_rows);
       const int64_t sbase = score_base(a, un, u);
-      for (int kt = kt0; kt < kt1; ++kt) {
+      for (int kt = kt0; kt < kt1; ++kt, ++pair) {
         const int t = kt * kTileKeys + kl;
         const bool fast = all_rows && (kt * kTileKeys + kTileKeys - 1 <= min_pos);
         const int ab = pair & 1;
+        if (ab != grp) continue;                   // the other group's tile
         ok = __all_sync(0xffffffffu, mbar_wait(&sh.acc_full[ab], (pair >> 1) & 1, sh.abort_flag, a.status));
         if (!ok) break;
         tc_fence_after();
@@ -1162,20 +1173,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             colsum += s;
           }
         }
-        ++pair;
-        // add the row parts of this key and write s(t)
-        if (part != 0) {
-          ok = mbar_wait(sh.red_empty, (xchg & 1) ^ 1, sh.abort_flag, a.status);
+        // add the group's two row halves of this key and write s(t)
+        if (gp != 0) {
+          ok = mbar_wait(&sh.red_empty[grp], (xchg & 1) ^ 1, sh.abort_flag, a.status);
           if (!ok) break;
-          sh.red[(part - 1) * kTileKeys + kl] = colsum;
-          mbar_arrive(sh.red_full);
+          sh.red[grp * kTileKeys + kl] = colsum;
+          mbar_arrive(&sh.red_full[grp]);
         } else {
-          ok = mbar_wait(sh.red_full, xchg & 1, sh.abort_flag, a.status);
+          ok = mbar_wait(&sh.red_full[grp], xchg & 1, sh.abort_flag, a.status);
           if (!ok) break;
-          float total = colsum;
-#pragma unroll
-          for (int x = 1; x < kParts; ++x) total += sh.red[(x - 1) * kTileKeys + kl];
-          mbar_arrive(sh.red_empty);
+          const float total = colsum + sh.red[grp * kTileKeys + kl];
+          mbar_arrive(&sh.red_empty[grp]);
           if (t < n) a.prepool[sbase + t] = total;
         }
         ++xchg;

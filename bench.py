@@ -128,15 +128,28 @@ class ClockSampler:
 # ------------------------------------------------------- algorithmic counts --
 
 def path_counts(w, B):
-    """Algorithmic bytes / flops per step of each kernel of the path (DESIGN
-    notes): K read once per pass, the window queries, the pre-pool score
-    written and read once, the kept K/V rows read and written, the kept index
-    written and read."""
+    """Algorithmic bytes / flops per step of each kernel of the path: K read
+    once, the queries, the pre-pool score written and read once, the kept K/V
+    rows read and written, the kept index written and read.  Variable-length
+    batches use their mean length (exact for the sums of per-token terms)."""
     U = w.L * w.b * w.Hkv
-    n = w.n
+    n = (sum(w.seqlens) / w.b) if w.varlen else w.n
     d = w.d
+    K = (sum(math.ceil(B * x) for x in w.seqlens) / w.b) if w.varlen else math.ceil(B * n)
+    if w.kind == "h2o":
+        causal = n * (n + 1) / 2                     # query-key pairs per head
+        flops = 2.0 * U * w.G * causal * d
+        qbytes = U * w.G * n * d * 2
+        kbytes = U * n * d * 2
+        return {
+            "pass1": {"bytes": kbytes + qbytes, "flops": flops},
+            "pass2": {"bytes": kbytes + qbytes + U * n * 4, "flops": flops},
+            "select": {"bytes": U * n * 4 + w.b * n + U * K * 4, "flops": 0.0},
+            "compact": {"bytes": U * K * 4 + 2 * 2 * U * K * d * 2, "flops": 0.0},
+            "path_bytes": kbytes + qbytes + U * n * 8 + U * K * 8 + 2 * 2 * U * K * d * 2 + w.b * n,
+            "kept": K,
+        }
     rows = w.G * w.W
-    K = math.ceil(B * n)
     kbytes = U * n * d * 2
     qbytes = U * rows * d * 2
     flops = 2.0 * U * rows * n * d
@@ -167,13 +180,12 @@ def run_gpu(args):
     w = I.WORKLOADS[args.workload]
     if args.layers:
         w = w.scaled(L=args.layers)
-    B = w.budgets[0]
-    if w.kind != "snapkv":
-        raise SystemExit("the bench times the SnapKV path")
+    B = args.budget if args.budget else w.budgets[0]
+    h2o = w.kind == "h2o"
 
     roles_np = I.workload_roles(w, seed=rank)
     K, V = I.make_kv(w, roles_np, seed=rank, device=dev)
-    qw = I.make_q_window(w, seed=rank, device=dev)
+    qw = I.make_q_full(w, seed=rank, device=dev) if h2o else I.make_q_window(w, seed=rank, device=dev)
     roles = torch.as_tensor(roles_np, device=dev)
     batch = R.Batch(w.L, w.b, w.Hq, w.Hkv, w.d, w.n, seqlens=list(w.seqlens) if w.varlen else None,
                     device=dev)
@@ -182,24 +194,32 @@ def run_gpu(args):
     keep = torch.empty(batch.kept_shape(B), dtype=torch.int32, device=dev)
     k_out = torch.empty(R.compact_shape(batch, B), dtype=torch.bfloat16, device=dev)
     v_out = torch.empty_like(k_out)
-    ws = R.workspace(R.OP_SNAPKV, batch, w.W, device=dev)
+    ws = R.workspace(R.OP_H2O if h2o else R.OP_SNAPKV, batch, w.W, device=dev)
     status = torch.zeros(1, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream(dev)
 
-    names = ["score", "select", "compact"]
+    names = ["pass1", "pass2", "select", "compact"] if h2o else ["score", "select", "compact"]
+    ns = len(names) - 2                              # score kernels
+
+    def score():
+        if h2o:
+            R.h2o_score(batch, qw, K, scores, ws=ws, status=status, stream=stream)
+        else:
+            # pool_k = 1: the pre-pool scores go straight out; the selector pools
+            R.snapkv_score(batch, qw, K, w.W, 1, scores, ws=ws, status=status, stream=stream)
 
     def step(ev=None):
-        # the path as three public calls: pre-pool scores (pool_k = 1 writes
-        # them straight out), selection with the pool fused, compaction
+        # the path as three public calls: scores, selection (pool fused),
+        # compaction
         if ev is not None:
-            R.set_stage_events(ev[1:2])
-        R.snapkv_score(batch, qw, K, w.W, 1, scores, ws=ws, status=status, stream=stream)
+            R.set_stage_events(ev[1:1 + ns])
+        score()
         if ev is not None:
-            R.set_stage_events(ev[2:3])
+            R.set_stage_events(ev[1 + ns:2 + ns])
         R.role_alloc_select(batch, scores, roles, params, keep, pool_k=w.pool_k, status=status,
                             stream=stream)
         if ev is not None:
-            R.set_stage_events(ev[3:4])
+            R.set_stage_events(ev[2 + ns:3 + ns])
         R.kv_compact(batch, K, V, keep, B, k_out, v_out, status=status, stream=stream)
         if ev is not None:
             R.set_stage_events([])
@@ -208,8 +228,9 @@ def run_gpu(args):
         step()
     torch.cuda.synchronize(dev)
 
-    # per-step events: [0] step start, [1] score kernel, [2] select, [3] compact
-    events = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    # per-step events: [0] step start, then one after each kernel
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(len(names) + 1)]
+              for _ in range(args.steps)]
     for evs in events:
         for e in evs:
             e.record(stream)       # create the underlying CUDA events
@@ -263,26 +284,29 @@ def run_gpu(args):
     roof["traffic"] = args.traffic
     roof["peak_source"] = peaks["source"] + " (burst)"
     path_frac = counts["path_bytes"] / (ms_step / 1e3) / 1e9 / peaks["hbm_gbs"]
+    tensor_util = {nm: counts[nm]["flops"] / (per_kernel[nm] / 1e3) / 1e12 / peaks["bf16_tflops"]
+                   for nm in names if counts[nm]["flops"] > 0}
 
     result = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": f"{w.name}: L={w.L} b={w.b} Hq={w.Hq} Hkv={w.Hkv} d={w.d} "
-                               f"N={w.n} W={w.W} pool={w.pool_k} B={B}",
+                               f"N={'varlen<=' if w.varlen else ''}{w.n} W={w.W} pool={w.pool_k} B={B}",
                    "global_batch": world * w.b, "seq_len": w.n, "parallelism": f"replicas x{world}",
-                   "l2": "inputs larger than L2 (17 GB K/V), no flush"},
+                   "l2": "inputs larger than L2, no flush"},
         "hbm_path_frac": path_frac,
+        "tensor_frac_of_measured_peak": tensor_util,
         "per_kernel_ms": per_kernel,
         "unit_tokens_per_s": world * w.L * w.Hkv * seq_tokens * args.steps / (elapsed_ms / 1e3),
         "roofline": roof,
         "clocks": clock_info,
-        "gpu_launches": 3 * args.steps,
+        "gpu_launches": len(names) * args.steps,
     }
 
     if not args.no_e2e:
-        result["e2e"] = run_e2e(args, w, B, batch, params, qw, K, V, roles, scores, keep, k_out,
-                                v_out, ws, status, stream, world, seq_tokens)
+        result["e2e"] = run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep,
+                                k_out, v_out, status, stream, world, seq_tokens)
     if rank == 0 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(w, B, args.cpu_seconds, host_inputs=(qw, K, V, roles_np))
     if rank == 0:
@@ -292,7 +316,7 @@ def run_gpu(args):
         dist.destroy_process_group()
 
 
-def run_e2e(args, w, B, batch, params, qw, K, V, roles, scores, keep, k_out, v_out, ws, status,
+def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_out, v_out, status,
             stream, world, seq_tokens):
     """The same step through the public calls with host buffers: the step's
     inputs are copied from pinned host memory and the kept indices and the
@@ -321,7 +345,7 @@ def run_e2e(args, w, B, batch, params, qw, K, V, roles, scores, keep, k_out, v_o
         K.copy_(h_k, non_blocking=True)
         V.copy_(h_v, non_blocking=True)
         roles.copy_(h_roles, non_blocking=True)
-        R.snapkv_score(batch, qw, K, w.W, 1, scores, ws=ws, status=status, stream=stream)
+        score()
         R.role_alloc_select(batch, scores, roles, params, keep, pool_k=w.pool_k, status=status,
                             stream=stream)
         R.kv_compact(batch, K, V, keep, B, k_out, v_out, status=status, stream=stream)
@@ -353,9 +377,13 @@ def oracle_units(w, B, units, qw_bits, k_bits, v_bits, roles_np):
     from paper_2607_13205_gb300 import inputs as I
 
     ob = O.Batch(w.L, w.b, w.Hq, w.Hkv, w.d, w.n, seqlens=list(w.seqlens) if w.varlen else None)
-    sc = O.snapkv_batch(ob, qw_bits, k_bits, w.W, w.pool_k, units=units)
-    sel = O.select_batch(ob, {u: sc[u][1] for u in sc}, roles_np, I.N_ROLES, I.PAPER_ALPHA,
-                         I.ROLE_KEY, 0.0, B)
+    if w.kind == "h2o":
+        sc = O.h2o_batch(ob, qw_bits, k_bits, units=units)
+        pooled = sc
+    else:
+        sc = O.snapkv_batch(ob, qw_bits, k_bits, w.W, w.pool_k, units=units)
+        pooled = {u: sc[u][1] for u in sc}
+    sel = O.select_batch(ob, pooled, roles_np, I.N_ROLES, I.PAPER_ALPHA, I.ROLE_KEY, 0.0, B)
     for u, (idx, _) in sel.items():
         O.compact_unit(ob.kv_rows(k_bits, u), idx)
         O.compact_unit(ob.kv_rows(v_bits, u), idx)
@@ -430,11 +458,11 @@ def run_reference(args):
     from paper_2607_13205_gb300 import inputs as I
 
     w = I.WORKLOADS[args.workload]
-    B = w.budgets[0]
+    B = args.budget if args.budget else w.budgets[0]
     w1 = w.scaled(L=1)
     roles_np = I.workload_roles(w1, seed=0)
     K, V = I.make_kv(w1, roles_np, seed=0, device="cpu")
-    qw = I.make_q_window(w1, seed=0, device="cpu")
+    qw = (I.make_q_full if w.kind == "h2o" else I.make_q_window)(w1, seed=0, device="cpu")
     qb, kb, vb = I.bf16_bits(qw), I.bf16_bits(K), I.bf16_bits(V)
     U = w.L * w.b * w.Hkv
     per_step = max(1, args.ref_units)
@@ -481,6 +509,7 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-units", type=int, default=2)
+    ap.add_argument("--budget", type=float, default=0.0, help="override the workload's budget")
     ap.add_argument("--layers", type=int, default=0,
                     help="override the layer count (smaller cases for profiling)")
     ap.add_argument("--traffic", type=float, default=None,

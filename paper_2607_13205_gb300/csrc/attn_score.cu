@@ -402,8 +402,8 @@ __device__ __forceinline__ void rowstats_epilogue(const ScoreArgs& a, const Work
     if (nrt == 1) a.partials[slot * kRowsMax + 128 + row] = make_float2(-INFINITY, 0.f);
   } else if (w.rb1 > w.rb0) {
     const int64_t o = (static_cast<int64_t>(w.u) * a.nrb_max + rb) * kRowsMax;
-    a.lse2[o + row] = (l > 0.f) ? m2 + __log2f(l) : INFINITY;
-    if (nrt == 1) a.lse2[o + 128 + row] = INFINITY;
+    a.lse2[o + row] = (l > 0.f) ? -(m2 + __log2f(l)) : -INFINITY;
+    if (nrt == 1) a.lse2[o + 128 + row] = -INFINITY;
   }
 }
 
@@ -464,12 +464,11 @@ __device__ __forceinline__ void colsum_epilogue(const ScoreArgs& a, const Work& 
         const float2 s2 = __fadd2_rn(__fadd2_rn(acc[0], acc[1]), __fadd2_rn(acc[2], acc[3]));
         colsum += s2.x + s2.y;
       } else {
-        const int32_t* pos = sh.pos + qslot * kRowsMax + j0;
         float s = 0.f;
 #pragma unroll
         for (int i = 0; i < NCOL; ++i) {
           const float e = fast_exp2(fmaf(__uint_as_float(r[i]), c1, nl[i]));
-          s += (t <= pos[i]) ? e : 0.f;
+          s += (t <= row_position(a, n, rb, j0 + i)) ? e : 0.f;
         }
         colsum += s;
       }
@@ -522,7 +521,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&sh.k_empty[i], 1);
     }
     for (int i = 0; i < C::SQ; ++i) {
-      mbar_init(&sh.q_full[i], 32);                     // every producer lane arrives
+      mbar_init(&sh.q_full[i], 1);
       mbar_init(&sh.q_empty[i], PASS == kPassColsum ? 1 + kEpiWarps * 32 : 1);
     }
     for (int i = 0; i < 2; ++i) {
@@ -590,17 +589,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = mbar_wait(&sh.q_empty[slot], ((qload / C::SQ) & 1) ^ 1, sh.abort_flag, a.status);
         ok = __shfl_sync(0xffffffffu, ok, 0);
         if (!ok) break;
-        if (PASS == kPassColsum) {
-          const int64_t lrow =
-              (static_cast<int64_t>(w.u) * (a.mode == kModeSnapKV ? 1 : a.nrb_max) + rb) * kRowsMax;
-          for (int j = lane; j < kRowsMax; j += 32) {
-            const int p = row_position(a, n, rb, j);
-            sh.pos[slot * kRowsMax + j] = p;
-            sh.lse[slot * kRowsMax + j] = (p >= 0) ? -a.lse2[lrow + j] : -INFINITY;
-          }
-        }
         if (lane == 0) {
-          mbar_arrive_expect_tx(&sh.q_full[slot], static_cast<uint32_t>(a.nrows) * D * 2);
+          const uint32_t nl_bytes = (PASS == kPassColsum) ? kRowsMax * 4 : 0;
+          mbar_arrive_expect_tx(&sh.q_full[slot], static_cast<uint32_t>(a.nrows) * D * 2 + nl_bytes);
+          if (PASS == kPassColsum) {
+            // the block's negated normalisers (-inf where a row does not exist)
+            const int64_t lrow =
+                (static_cast<int64_t>(w.u) * (a.mode == kModeSnapKV ? 1 : a.nrb_max) + rb) * kRowsMax;
+            bulk_copy_g2s(sh.lse + slot * kRowsMax, a.lse2 + lrow, nl_bytes, &sh.q_full[slot]);
+          }
           uint8_t* dst = sh.q + slot * C::kQSlotBytes;
           const bool window = (a.mode == kModeSnapKV);
           const int64_t t0 = window ? 0 : static_cast<int64_t>(rb) * a.P;
@@ -612,8 +609,6 @@ __global__ void __launch_bounds__(kThreads, 1)
               tma_load_2d(dst + hf * C::kQHalfBytes + g * a.P * 128, &q_map, c.x + hf * 64, c.y,
                           &sh.q_full[slot]);
           }
-        } else {
-          mbar_arrive(&sh.q_full[slot]);
         }
         ++qload;
       }
@@ -803,12 +798,14 @@ __device__ __forceinline__ int ld_acquire_gpu(const int32_t* p) {
   return v;
 }
 
-// Key-tile range of chunk c of a unit with n keys.
+// Key-tile range of chunk c of a unit with n keys: the unit's tiles split as
+// evenly as possible over its n_chunks chunks (sequences of a varlen batch
+// keep their whole gang busy).
 __device__ __forceinline__ void chunk_tiles(const ScoreArgs& a, int n, int c, int* kt0, int* kt1) {
   const int ntiles = (n + kTileKeys - 1) / kTileKeys;
-  *kt0 = c * a.chunk_tiles;
-  *kt1 = min(ntiles, *kt0 + a.chunk_tiles);
-  if (*kt1 < *kt0) *kt1 = *kt0;
+  const int ct = (ntiles + a.n_chunks - 1) / a.n_chunks;
+  *kt0 = min(ntiles, c * ct);
+  *kt1 = min(ntiles, *kt0 + ct);
 }
 
 template <int D>
@@ -1230,7 +1227,7 @@ __global__ void snapkv_lse_kernel(const ScoreArgs a, const float* __restrict__ l
       }
     }
   }
-  a.lse2[static_cast<int64_t>(u) * kRowsMax + j] = out;
+  a.lse2[static_cast<int64_t>(u) * kRowsMax + j] = -out;
 }
 
 // Stride-1 max-pool over each unit's score row, truncated at the sequence

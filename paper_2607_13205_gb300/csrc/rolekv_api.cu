@@ -564,6 +564,8 @@ int role_alloc_select(const rolekv_batch* batch, const float* scores, const uint
   if (rc) return rc;
   if (scores == nullptr || roles == nullptr || keep_idx == nullptr)
     return fail(ROLEKV_ERR_INVALID_ARG, "scores, roles and keep_idx are required");
+  if ((reinterpret_cast<uintptr_t>(scores) & 3u) || (reinterpret_cast<uintptr_t>(keep_idx) & 3u))
+    return fail(ROLEKV_ERR_INVALID_ARG, "scores and keep_idx must be 4-byte aligned");
   if (pool_k < 1 || pool_k > 15 || pool_k % 2 == 0)
     return fail(ROLEKV_ERR_UNSUPPORTED, "pool_k=%d must be odd, 1..15", pool_k);
   SelectArgs a;

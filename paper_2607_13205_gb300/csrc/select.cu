@@ -1,9 +1,31 @@
 // Role-conditional allocation and per-bucket top-k (Section 4.1, Algorithm 1):
 // pool the scores (optional), count the roles, split the budget ceil(B n)
 // across role buckets, and keep the top-q_r tokens of every bucket, ties to the
-// lower index.  One CTA per (layer, sequence, KV head) holds the whole score
-// row in shared memory; everything after the fp32 -> ordered-key mapping is
+// lower index.  One CTA per (layer, sequence, KV head) holds the unit's keys
+// in shared memory; everything after the fp32 -> ordered-key mapping is
 // integer, so the kept set is bit-exact for a given score row.
+//
+// Slots.  Shared memory holds the unit in "slots": slot s is token s - off,
+// where off = (start address of the score row / 4) mod 4, so that every group
+// of four slots is one aligned 16-byte vector both in global and in shared
+// memory.  Slots outside [off, off + n) have role 0xFF and are never kept.
+//
+// The threshold of each bucket is found by a radix descent over the keys'
+// bits, most significant first:
+//   pass 1  load, pool, key; role counts and, per role, a histogram of the
+//           key's bits 30..31-NB (the top bit is shared by every key when all
+//           scores have one sign): exponent and leading mantissa bits.
+//   quotas  one warp, lane r for role r (water-filling, largest remainders).
+//   first digit from the pass-1 histograms, per bucket.
+//   pass 2  every token is decided (kept / dropped) unless its first digit is
+//           its bucket's threshold digit; those "candidates" (a few percent)
+//           go to a list in shared memory.
+//   list    the remaining bits in 8-bit rounds over the list; ties at the
+//           threshold are ranked in index order; the kept ones join the bits.
+// A unit with a NaN, keys of both signs, or more candidates than the list
+// holds takes the general path: four 8-bit rounds over all slots.
+// Kept positions are then written in ascending order from a block-wide scan
+// of the bit words.
 #include <cuda_runtime.h>
 
 #include <cmath>
@@ -15,10 +37,23 @@
 namespace rolekv {
 namespace {
 
-constexpr int kThreads = 1024;
-constexpr int kWarps = kThreads / 32;
-constexpr int kMaxPerThread = (ROLEKV_SELECT_MAX_N + kThreads - 1) / kThreads;
 constexpr int kR = ROLEKV_MAX_ROLES;
+constexpr uint32_t kCodeKeep = 0x40;   // the token's bucket keeps everything
+constexpr uint32_t kCodeDrop = 0x80;   // no bucket keeps the token
+// codes 0 .. kR-1: the token's bucket keeps only keys above a threshold
+constexpr int kTieCap = 256;           // ranked ties held in shared memory
+
+// Groups (of four slots) reserved per CTA: n_max tokens plus up to three
+// leading slots, rounded to a multiple of 32 groups so that the bit words
+// (one per 8 groups) end on a 16-byte boundary.
+__host__ __device__ inline int select_groups(int n_max) { return (((n_max + 3 + 3) / 4) + 31) & ~31; }
+// Width of the first digit: 2^NB bins per role.
+__host__ __device__ inline int first_digit_bits(int n_max) { return n_max > 16384 ? 11 : 10; }
+// Bytes of the region that holds the pass-1 histograms (8 roles x 2^NB bins
+// x 16-bit counts), reused for the candidate list (4-byte entries).
+__host__ __device__ inline size_t region_bytes(int n_max) {
+  return static_cast<size_t>(kR) * (size_t{1} << first_digit_bits(n_max)) * 2;
+}
 
 // Monotone map of a float to uint32 (larger float -> larger key); -0 is folded
 // onto +0 so equal floats give equal keys.
@@ -28,20 +63,18 @@ __device__ __forceinline__ uint32_t ordered_key(float f) {
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
-struct SelShared {
-  int64_t quota[kR];
-  int64_t size[kR];
-  int32_t bucket_of_role[256];
-  uint32_t prefix[kR];
-  uint32_t need[kR];
-  int32_t mode[kR];              // 0 none kept, 1 all kept, 2 threshold
-  int32_t hist[kR][256];
-  int32_t warp_cnt[kWarps][kR];  // per-warp tie counts, then exclusive bases
-  int32_t warp_kept[kWarps];
-  int32_t kept_role[kR];
-  int64_t keep_off;
-  int32_t nonfinite;
-};
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// x << s, with every shift of 64 or more giving 0 (PTX clamps the amount).
+__device__ __forceinline__ uint64_t shl64(uint64_t x, uint32_t s) {
+  uint64_t r;
+  asm("shl.b64 %0, %1, %2;" : "=l"(r) : "l"(x), "r"(s));
+  return r;
+}
 
 __device__ __forceinline__ int warp_sum(int v) {
 #pragma unroll
@@ -49,69 +82,351 @@ __device__ __forceinline__ int warp_sum(int v) {
   return v;
 }
 
-// Integer quotas of one sequence; the same arithmetic as the public
-// description in rolekv.h (water-filling then largest remainder).
-__device__ void compute_quotas(const SelectArgs& a, const int64_t* count, int64_t K_full,
-                               int64_t* q) {
-  for (int r = 0; r < kR; ++r) q[r] = 0;
-  const int R = a.n_roles;
-  if (a.policy == ROLEKV_POLICY_GLOBAL) {
-    int64_t elig = 0;
-    for (int r = 0; r < R; ++r)
-      if (!((a.ban_mask >> r) & 1u)) elig += count[r];
-    q[0] = K_full < elig ? K_full : elig;
-    return;
+__device__ __forceinline__ int64_t warp_sum64(int64_t v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+struct SelShared {
+  int64_t keep_off;
+  int32_t count[kR];       // tokens per role
+  int32_t quota[kR];       // q_b per bucket
+  uint32_t prefix[kR];     // threshold key bits found so far
+  int32_t need[kR];        // tokens equal to the prefix still to keep
+  uint32_t thr[kR];        // keep iff key >= thr (ties ranked apart when partial)
+  int32_t mode[kR];        // 0 none kept, 1 all kept, 2 threshold
+  int32_t cand[kR];        // candidates after the first digit
+  int32_t code_of_role[256];
+  int32_t hist[kR][256];
+  int32_t warp_tot[32];
+  int32_t kept_role[kR];
+  uint32_t ties[kTieCap];  // (bucket << 16) | slot of keys equal to a threshold
+  uint32_t top_and, top_or;
+  int32_t list_n, tie_n;
+  int32_t nan_hint;        // a sum of the unit's scores was NaN
+  int32_t nan_seen;        // a pooled window held a NaN
+  int32_t any_threshold;
+  int32_t general;         // take the full-pass descent
+  uint32_t partial_ties;   // buckets with more threshold ties than slots left
+};
+
+// Slots 4g .. 4g+3 of a score row; slots outside [off, off + n) read -inf.
+// sp + (4g - off) is 16-byte aligned by the choice of off.
+__device__ __forceinline__ float4 load_slots(const float* sp, int off, int n, int g) {
+  const int s0 = 4 * g - off;
+  if (s0 >= 0 && s0 + 4 <= n) return __ldg(reinterpret_cast<const float4*>(sp + s0));
+  float4 r;
+  r.x = (s0 >= 0 && s0 < n) ? __ldg(sp + s0) : -INFINITY;
+  r.y = (s0 + 1 >= 0 && s0 + 1 < n) ? __ldg(sp + s0 + 1) : -INFINITY;
+  r.z = (s0 + 2 >= 0 && s0 + 2 < n) ? __ldg(sp + s0 + 2) : -INFINITY;
+  r.w = (s0 + 3 >= 0 && s0 + 3 < n) ? __ldg(sp + s0 + 3) : -INFINITY;
+  return r;
+}
+
+// Role bytes of slots 4g .. 4g+3 (0xFF outside the sequence).
+__device__ __forceinline__ uint32_t load_roles(const uint8_t* rp, int off, int n, int g, bool vec) {
+  const int s0 = 4 * g - off;
+  if (vec && s0 >= 0 && s0 + 4 <= n) return __ldg(reinterpret_cast<const uint32_t*>(rp + s0));
+  uint32_t w = 0;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const int t = s0 + j;
+    const uint32_t r = (t >= 0 && t < n) ? static_cast<uint32_t>(__ldg(rp + t)) : 0xFFu;
+    w |= r << (8 * j);
   }
-  bool live[kR];
-  int64_t elig = 0;
-  for (int r = 0; r < kR; ++r) {
-    live[r] = (r < R) && a.alpha_fx[r] > 0 && count[r] > 0;
-    if (live[r]) elig += count[r];
-  }
-  const int64_t K = K_full < elig ? K_full : elig;
-  int64_t left = K;
-  bool changed = true;
-  while (changed) {
-    changed = false;
-    int64_t A = 0;
-    for (int r = 0; r < kR; ++r)
-      if (live[r]) A += a.alpha_fx[r];
-    if (A == 0) break;
-    bool sat[kR];
-    for (int r = 0; r < kR; ++r) sat[r] = live[r] && a.alpha_fx[r] * left >= count[r] * A;
-    for (int r = 0; r < kR; ++r)
-      if (sat[r]) {
-        q[r] = count[r];
-        live[r] = false;
-        changed = true;
-      }
-    for (int r = 0; r < kR; ++r)
-      if (sat[r]) left -= count[r];
-  }
-  int64_t A = 0;
-  for (int r = 0; r < kR; ++r)
-    if (live[r]) A += a.alpha_fx[r];
-  if (A == 0) return;
-  int64_t rem[kR];
-  int64_t given = 0;
-  for (int r = 0; r < kR; ++r)
-    if (live[r]) {
-      q[r] = (a.alpha_fx[r] * left) / A;
-      rem[r] = (a.alpha_fx[r] * left) % A;
-      given += q[r];
+  return w;
+}
+
+struct UnitView {
+  const float* sp;
+  const uint8_t* rp;
+  int off, n, ngroups;
+  bool rvec;
+};
+
+// Pass 1 for a pool half-width HW known at compile time.
+template <int HW, int NT>
+__device__ __forceinline__ void pass1(const UnitView& v, int n_roles, int nb, uint4* keys4,
+                                      uint32_t* hist16, uint64_t& rc, bool& nan_hint,
+                                      uint32_t& top_and, uint32_t& top_or) {
+  constexpr int NB = (HW + 3) / 4;   // neighbour groups on each side
+  const int sh0 = 31 - nb;
+  const uint32_t bmask = (1u << nb) - 1u;
+  const int words_per_role = 1 << (nb - 1);
+  for (int g = threadIdx.x; g < v.ngroups; g += NT) {
+    float x[4 * (2 * NB + 1)];
+#pragma unroll
+    for (int o = -NB; o <= NB; ++o) {
+      const float4 f = load_slots(v.sp, v.off, v.n, g + o);
+      x[4 * (o + NB) + 0] = f.x;
+      x[4 * (o + NB) + 1] = f.y;
+      x[4 * (o + NB) + 2] = f.z;
+      x[4 * (o + NB) + 3] = f.w;
     }
-  int64_t extra = left - given;
-  while (extra > 0) {
-    int best = -1;
-    for (int r = 0; r < kR; ++r)
-      if (live[r] && (best < 0 || rem[r] > rem[best])) best = r;
-    q[best] += 1;
-    live[best] = false;
-    --extra;
+    const float* c = x + 4 * NB;
+    const float sum = (c[0] + c[1]) + (c[2] + c[3]);
+    nan_hint |= (sum != sum);
+    uint32_t k[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      float m = c[j - HW];
+#pragma unroll
+      for (int o = -HW + 1; o <= HW; o += 2) {
+        if (o < HW)
+          m = max3f(m, c[j + o], c[j + o + 1]);
+        else
+          m = fmaxf(m, c[j + o]);
+      }
+      k[j] = ordered_key(m);
+    }
+    keys4[g] = make_uint4(k[0], k[1], k[2], k[3]);
+    const uint32_t rw = load_roles(v.rp, v.off, v.n, g, v.rvec);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint32_t r = (rw >> (8 * j)) & 0xFFu;
+      rc += shl64(1ull, 8u * r);
+      if (r < static_cast<uint32_t>(n_roles)) {
+        top_and &= k[j];
+        top_or |= k[j];
+        const uint32_t bin = (k[j] >> sh0) & bmask;
+        atomicAdd(&hist16[r * words_per_role + (bin >> 1)], 1u << (16 * (bin & 1u)));
+      }
+    }
   }
 }
 
-__global__ void __launch_bounds__(kThreads, 1) select_kernel(const SelectArgs a) {
+// Quotas of one sequence by warp 0, lane r for role r: water-filling of the
+// weights over the role counts, then the integer remainders to the largest
+// fractional parts (ties to the lower role), the arithmetic stated in rolekv.h.
+__device__ void quotas_warp(const SelectArgs& a, int lane, int64_t K_full, SelShared& S) {
+  const int r = lane;
+  const bool valid = r < a.n_roles;
+  const bool banned = valid && ((a.ban_mask >> r) & 1u);
+  const int64_t cnt = valid ? S.count[r] : 0;
+  const int64_t alpha = r < kR ? a.alpha_fx[r] : 0;
+  int64_t q = 0, bsize = 0;
+  if (a.policy == ROLEKV_POLICY_GLOBAL) {
+    const int64_t elig = warp_sum64((valid && !banned) ? cnt : 0);
+    if (r == 0) {
+      q = K_full < elig ? K_full : elig;
+      bsize = elig;
+    }
+  } else {
+    bool live = valid && alpha > 0 && cnt > 0;
+    const int64_t elig = warp_sum64(live ? cnt : 0);
+    int64_t left = K_full < elig ? K_full : elig;
+    for (int it = 0; it <= kR; ++it) {
+      const int64_t A = warp_sum64(live ? alpha : 0);
+      if (A == 0) break;
+      const bool sat = live && alpha * left >= cnt * A;
+      if (!__any_sync(0xffffffffu, sat)) break;
+      if (sat) {
+        q = cnt;
+        live = false;
+      }
+      left -= warp_sum64(sat ? cnt : 0);
+    }
+    const int64_t A = warp_sum64(live ? alpha : 0);
+    int64_t rem = -1;
+    if (live && A != 0) {
+      q = alpha * left / A;
+      rem = alpha * left % A;
+    }
+    const int64_t extra = left - warp_sum64(live ? q : 0);
+    int rank = 0;
+#pragma unroll
+    for (int x = 0; x < kR; ++x) {
+      const int64_t rx = __shfl_sync(0xffffffffu, rem, x);
+      const int lx = __shfl_sync(0xffffffffu, static_cast<int>(live), x);
+      if (lx && (rx > rem || (rx == rem && x < r))) ++rank;
+    }
+    if (live && A != 0 && rank < extra) q += 1;
+    bsize = cnt;
+  }
+  int mode = 0;
+  if (r < kR) {
+    mode = (q <= 0) ? 0 : (q >= bsize ? 1 : 2);
+    S.quota[r] = static_cast<int32_t>(q);
+    S.mode[r] = mode;
+    S.prefix[r] = 0;
+    S.need[r] = static_cast<int32_t>(q);
+    S.thr[r] = 0xFFFFFFFFu;   // above every key; set by the last radix round
+    S.cand[r] = 0;
+  }
+  const bool any = __any_sync(0xffffffffu, mode == 2);
+  if (lane == 0) {
+    S.any_threshold = any;
+    S.partial_ties = 0;
+    S.list_n = 0;
+    S.tie_n = 0;
+  }
+}
+
+// The bucket's key among its remaining candidates with need[b] keys at or
+// above it: warp b reads the histogram of the digit at `shift` (clearing it),
+// finds the digit where the count from the top reaches need[b], appends it to
+// prefix[b] and subtracts the keys above.  At shift 0 the prefix is the
+// q_b-th largest key; thr[b] and the partial-tie flag are then set.
+__device__ void descend(SelShared& S, int b, int lane, int shift) {
+  int c[8];
+  int mine = 0;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    c[i] = S.hist[b][lane * 8 + i];
+    S.hist[b][lane * 8 + i] = 0;
+    mine += c[i];
+  }
+  int incl = mine;   // tokens whose digit is in this lane's range or above
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int v = __shfl_down_sync(0xffffffffu, incl, o);
+    if (lane + o < 32) incl += v;
+  }
+  const int above = incl - mine;
+  const int need = S.need[b];
+  int found = -1, gt_before = 0, at_digit = 0;
+  if (above < need && above + mine >= need) {
+    int acc = above;
+#pragma unroll
+    for (int i = 7; i >= 0; --i) {
+      if (found < 0 && acc + c[i] >= need) {
+        found = lane * 8 + i;
+        gt_before = acc;
+        at_digit = c[i];
+      }
+      acc += c[i];
+    }
+  }
+  const unsigned who = __ballot_sync(0xffffffffu, found >= 0);
+  const int src = who ? __ffs(who) - 1 : 0;
+  const int fd = __shfl_sync(0xffffffffu, found, src);
+  const int gb = __shfl_sync(0xffffffffu, gt_before, src);
+  const int ad = __shfl_sync(0xffffffffu, at_digit, src);
+  if (lane == 0 && who != 0) {
+    const uint32_t prefix = S.prefix[b] | (static_cast<uint32_t>(fd) << shift);
+    const int need2 = need - gb;
+    S.prefix[b] = prefix;
+    S.need[b] = need2;
+    if (shift == 0) {
+      // ad keys of the bucket equal the threshold; need2 of them are kept
+      S.thr[b] = (need2 >= ad) ? prefix : prefix + 1u;
+      if (need2 < ad) atomicOr(&S.partial_ties, 1u << b);
+    }
+  }
+}
+
+// First digit (bits 30..31-nb, the shared top bit above them) of bucket b from
+// the per-role 16-bit histograms of pass 1; the bucket's histogram is the sum
+// over its roles.
+__device__ void descend_first(const SelectArgs& a, SelShared& S, const uint32_t* hist16, int b,
+                              int lane, int nb) {
+  const int bpl = 1 << (nb - 5);   // bins per lane
+  const int wpr = 1 << (nb - 1);   // words per role
+  const uint32_t roles = (a.policy == ROLEKV_POLICY_GLOBAL)
+                             ? (((1u << a.n_roles) - 1u) & ~a.ban_mask)
+                             : (1u << b);
+  auto count = [&](int bin) {
+    int s = 0;
+    for (uint32_t m = roles; m != 0; m &= m - 1) {
+      const int r = __ffs(m) - 1;
+      s += static_cast<int>((hist16[r * wpr + (bin >> 1)] >> (16 * (bin & 1))) & 0xFFFFu);
+    }
+    return s;
+  };
+  int mine = 0;
+  for (int i = 0; i < bpl; ++i) mine += count(lane * bpl + i);
+  int incl = mine;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int v = __shfl_down_sync(0xffffffffu, incl, o);
+    if (lane + o < 32) incl += v;
+  }
+  const int above = incl - mine;
+  const int need = S.need[b];
+  int found = -1, gt_before = 0, at_digit = 0;
+  if (above < need && above + mine >= need) {
+    int acc = above;
+    for (int i = bpl - 1; i >= 0; --i) {
+      const int ci = count(lane * bpl + i);
+      if (acc + ci >= need) {
+        found = lane * bpl + i;
+        gt_before = acc;
+        at_digit = ci;
+        break;
+      }
+      acc += ci;
+    }
+  }
+  const unsigned who = __ballot_sync(0xffffffffu, found >= 0);
+  const int src = who ? __ffs(who) - 1 : 0;
+  const int fd = __shfl_sync(0xffffffffu, found, src);
+  const int gb = __shfl_sync(0xffffffffu, gt_before, src);
+  const int ad = __shfl_sync(0xffffffffu, at_digit, src);
+  if (lane == 0) {
+    if (who == 0) {
+      S.general = 1;   // counts disagree with the quota: let the full path decide
+    } else {
+      const int sh0 = 31 - nb;
+      S.prefix[b] = (S.top_and & 0x80000000u) | (static_cast<uint32_t>(fd) << sh0);
+      S.need[b] = need - gb;
+      S.cand[b] = ad;
+    }
+  }
+}
+
+// Exclusive prefix, in slot order, of popc(mask_of(q)) over the bit words
+// q < nwords: warp w walks a contiguous range of words (a multiple of 32), the
+// warps' totals are combined through shared memory, and body(q, mask, rank of
+// the word's first set bit) runs once per word.  Returns the total.  Every
+// thread of the CTA must call it.
+template <int NT, class MaskF, class BodyF>
+__device__ int scan_words(int nwords, MaskF mask_of, BodyF body, int32_t* warp_tot) {
+  constexpr int NW = NT / 32;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int wseg = ((nwords + NW - 1) / NW + 31) & ~31;
+  const int q_begin = warp * wseg;
+  const int q_end = min(nwords, q_begin + wseg);
+  int tot = 0;
+  for (int q0 = q_begin; q0 < q_end; q0 += 32) {
+    const int q = q0 + lane;
+    if (q < q_end) tot += __popc(mask_of(q));
+  }
+  tot = warp_sum(tot);
+  if (lane == 0) warp_tot[warp] = tot;
+  __syncthreads();
+  int base = warp_sum(lane < warp ? warp_tot[lane] : 0);
+  const int total = warp_sum(lane < NW ? warp_tot[lane] : 0);
+  for (int q0 = q_begin; q0 < q_end; q0 += 32) {
+    const int q = q0 + lane;
+    const uint32_t m = q < q_end ? mask_of(q) : 0u;
+    const int c = __popc(m);
+    int incl = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    if (q < q_end) body(q, m, base + incl - c);
+    base += __shfl_sync(0xffffffffu, incl, 31);
+  }
+  __syncthreads();
+  return total;
+}
+
+// Keep bits of slots 4g .. 4g+3 (bit j = slot 4g+j) packed into one 32-bit
+// word per 8 lanes; the lane with (lane & 7) == 0 stores word g / 8.
+__device__ __forceinline__ void store_bits(uint32_t* bits, int g, int nwords, int lane, uint32_t m4) {
+  uint32_t x = m4 << (4 * (lane & 7));
+  x |= __shfl_xor_sync(0xffffffffu, x, 1);
+  x |= __shfl_xor_sync(0xffffffffu, x, 2);
+  x |= __shfl_xor_sync(0xffffffffu, x, 4);
+  if ((lane & 7) == 0 && g < 8 * nwords) bits[g >> 3] = x;
+}
+
+template <int NT>
+__global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs a) {
+  constexpr int NW = NT / 32;
   extern __shared__ __align__(16) uint8_t dyn[];
   __shared__ SelShared S;
   const int tid = threadIdx.x;
@@ -134,338 +449,404 @@ __global__ void __launch_bounds__(kThreads, 1) select_kernel(const SelectArgs a)
   const int64_t rbase = a.varlen ? tok0 : static_cast<int64_t>(s) * a.n_max;
   const int64_t K_s = kept_slots(n, a.budget_fx);
 
-  uint32_t* keys = reinterpret_cast<uint32_t*>(dyn);
-  uint8_t* roles = dyn + static_cast<size_t>(a.n_max) * 4;
-  uint32_t* keptbits = reinterpret_cast<uint32_t*>(roles + ((a.n_max + 15) & ~15));
+  UnitView v;
+  v.sp = a.scores + sbase;
+  v.rp = a.roles + rbase;
+  v.off = static_cast<int>((reinterpret_cast<uintptr_t>(v.sp) >> 2) & 3);
+  v.n = n;
+  const int nslots = v.off + n;
+  v.ngroups = (nslots + 3) >> 2;
+  v.rvec = ((reinterpret_cast<uintptr_t>(v.rp) - static_cast<uintptr_t>(v.off)) & 3u) == 0;
+  const int off = v.off, ngroups = v.ngroups;
+  const int nwords = (nslots + 31) >> 5;
+  const int iters = (ngroups + NT - 1) / NT;
+  const int nb = first_digit_bits(a.n_max);
+  const int groups_alloc = select_groups(a.n_max);
+  uint4* keys4 = reinterpret_cast<uint4*>(dyn);
+  const uint32_t* keys = reinterpret_cast<const uint32_t*>(keys4);
+  uint32_t* bits = reinterpret_cast<uint32_t*>(dyn + static_cast<size_t>(groups_alloc) * 16);
+  uint32_t* region = bits + groups_alloc / 8;   // 16-byte aligned (groups_alloc % 32 == 0)
+  uint32_t* hist16 = region;                    // pass 1 histograms
+  uint32_t* list = region;                      // then the candidate list
+  const int list_cap = static_cast<int>(region_bytes(a.n_max) / 4);
 
-  // ---- offsets of this unit's kept row
   if (tid < kR) {
+    S.count[tid] = 0;
     S.kept_role[tid] = 0;
   }
-  if (tid == 0) S.nonfinite = 0;
+  if (tid == 0) {
+    S.nan_hint = 0;
+    S.nan_seen = 0;
+    S.general = 0;
+    S.top_and = 0xFFFFFFFFu;
+    S.top_or = 0u;
+  }
+  for (int x = tid; x < kR * 256; x += NT) (&S.hist[0][0])[x] = 0;
+  {
+    uint4* r4 = reinterpret_cast<uint4*>(region);
+    const int n4 = static_cast<int>(region_bytes(a.n_max) / 16);
+    for (int x = tid; x < n4; x += NT) r4[x] = make_uint4(0u, 0u, 0u, 0u);
+  }
+
+  // ---- offset of this unit's kept row
   {
     int64_t part = 0;
     if (a.varlen) {
-      for (int x = tid; x < s; x += kThreads)
+      for (int x = tid; x < s; x += NT)
         part += kept_slots(a.cu_seqlens[x + 1] - a.cu_seqlens[x], a.budget_fx);
     }
-    // block reduction of `part` through the warp_kept scratch
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
-    __shared__ int64_t red64[kWarps];
+    __shared__ int64_t red64[NW];
     if (lane == 0) red64[warp] = part;
     __syncthreads();
     if (tid == 0) {
       int64_t cu = 0;
-      for (int w = 0; w < kWarps; ++w) cu += red64[w];
+      for (int w = 0; w < NW; ++w) cu += red64[w];
       S.keep_off = a.varlen ? (static_cast<int64_t>(l) * a.Hkv + h) * a.Ktot + cu
                             : static_cast<int64_t>(u) * a.K_dense;
     }
   }
 
-  // ---- load roles and scores, pool, map to ordered keys
-  for (int t = tid; t < n; t += kThreads) roles[t] = a.roles[rbase + t];
-  if (a.pool_k <= 1) {
-    for (int t = tid; t < n; t += kThreads) {
-      const float f = a.scores[sbase + t];
-      if (isnan(f)) S.nonfinite = 1;
-      keys[t] = isnan(f) ? 0u : ordered_key(f);
-    }
-  } else {
-    for (int t = tid; t < n; t += kThreads) keys[t] = __float_as_uint(a.scores[sbase + t]);
-    __syncthreads();
-    float pooled[kMaxPerThread];
-    const int hw = a.pool_k / 2;
-#pragma unroll
-    for (int i = 0; i < kMaxPerThread; ++i) {
-      const int t = tid + i * kThreads;
-      float m = 0.f;
-      if (t < n) {
-        const int lo = max(0, t - hw), hi = min(n - 1, t + hw);
-        m = __uint_as_float(keys[lo]);
-        bool nan_seen = isnan(m);
-        for (int x = lo + 1; x <= hi; ++x) {
-          const float v = __uint_as_float(keys[x]);
-          nan_seen |= isnan(v);
-          m = fmaxf(m, v);
-        }
-        if (nan_seen) {
-          S.nonfinite = 1;
-          m = NAN;
-        }
-      }
-      pooled[i] = m;
-    }
-    __syncthreads();
-#pragma unroll
-    for (int i = 0; i < kMaxPerThread; ++i) {
-      const int t = tid + i * kThreads;
-      if (t < n) keys[t] = isnan(pooled[i]) ? 0u : ordered_key(pooled[i]);
-    }
-  }
-
-  // ---- role counts
+  // ---- pass 1: load, pool, key, role counts, first-digit histograms
   {
-    int cnt[kR];
-#pragma unroll
-    for (int r = 0; r < kR; ++r) cnt[r] = 0;
-    for (int t = tid; t < n; t += kThreads) {
-      const int r = roles[t];
-#pragma unroll
-      for (int x = 0; x < kR; ++x) cnt[x] += (r == x);
+    uint64_t rc = 0;
+    bool nan_hint = false;
+    uint32_t tand = 0xFFFFFFFFu, tor = 0u;
+    switch (a.pool_k >> 1) {
+      case 0: pass1<0, NT>(v, a.n_roles, nb, keys4, hist16, rc, nan_hint, tand, tor); break;
+      case 1: pass1<1, NT>(v, a.n_roles, nb, keys4, hist16, rc, nan_hint, tand, tor); break;
+      case 2: pass1<2, NT>(v, a.n_roles, nb, keys4, hist16, rc, nan_hint, tand, tor); break;
+      case 3: pass1<3, NT>(v, a.n_roles, nb, keys4, hist16, rc, nan_hint, tand, tor); break;
+      case 4: pass1<4, NT>(v, a.n_roles, nb, keys4, hist16, rc, nan_hint, tand, tor); break;
+      case 5: pass1<5, NT>(v, a.n_roles, nb, keys4, hist16, rc, nan_hint, tand, tor); break;
+      case 6: pass1<6, NT>(v, a.n_roles, nb, keys4, hist16, rc, nan_hint, tand, tor); break;
+      default: pass1<7, NT>(v, a.n_roles, nb, keys4, hist16, rc, nan_hint, tand, tor); break;
     }
-    if (tid < kR) S.size[tid] = 0;
-    __syncthreads();
 #pragma unroll
     for (int r = 0; r < kR; ++r) {
-      const int v = warp_sum(cnt[r]);
-      if (lane == 0 && v) atomicAdd(reinterpret_cast<unsigned long long*>(&S.size[r]),
-                                    static_cast<unsigned long long>(v));
+      const int c = warp_sum(static_cast<int>((rc >> (8 * r)) & 0xFFu));
+      if (lane == 0 && c) atomicAdd(&S.count[r], c);
     }
-    __syncthreads();
-  }
-
-  // ---- quotas and bucket sizes
-  if (tid == 0) {
-    int64_t count[kR];
-    for (int r = 0; r < kR; ++r) count[r] = (r < a.n_roles) ? S.size[r] : 0;
-    int64_t q[kR];
-    compute_quotas(a, count, K_s, q);
-    int64_t bsize[kR];
-    for (int r = 0; r < kR; ++r) bsize[r] = 0;
-    if (a.policy == ROLEKV_POLICY_GLOBAL) {
-      for (int r = 0; r < a.n_roles; ++r)
-        if (!((a.ban_mask >> r) & 1u)) bsize[0] += count[r];
-    } else {
-      for (int r = 0; r < kR; ++r) bsize[r] = count[r];
+    tand = __reduce_and_sync(0xffffffffu, tand);
+    tor = __reduce_or_sync(0xffffffffu, tor);
+    const bool nh = __any_sync(0xffffffffu, nan_hint);
+    if (lane == 0) {
+      atomicAnd(&S.top_and, tand);
+      atomicOr(&S.top_or, tor);
+      if (nh) S.nan_hint = 1;
     }
-    for (int r = 0; r < kR; ++r) {
-      S.quota[r] = q[r];
-      S.size[r] = bsize[r];
-      S.mode[r] = (q[r] <= 0) ? 0 : (q[r] >= bsize[r] ? 1 : 2);
-      S.prefix[r] = 0;
-      S.need[r] = static_cast<uint32_t>(q[r]);
-    }
-  }
-  for (int x = tid; x < 256; x += kThreads) {
-    int b = -1;
-    if (x < a.n_roles && !((a.ban_mask >> x) & 1u))
-      b = (a.policy == ROLEKV_POLICY_GLOBAL) ? 0 : x;
-    S.bucket_of_role[x] = b;
   }
   __syncthreads();
 
-  // ---- radix threshold per bucket: 4 rounds of 8-bit digits, most
-  // significant first; after them prefix[b] is the q_b-th largest key of the
-  // bucket and need[b] the number of tokens equal to it that are kept.
-  bool any_threshold = false;
-#pragma unroll
-  for (int r = 0; r < kR; ++r) any_threshold |= (S.mode[r] == 2);
-  if (any_threshold) {
-    for (int round = 0; round < 4; ++round) {
-      const int shift = 24 - 8 * round;
-      const uint32_t hi_mask = (round == 0) ? 0u : (0xFFFFFFFFu << (shift + 8));
-      for (int x = tid; x < kR * 256; x += kThreads) (&S.hist[0][0])[x] = 0;
-      __syncthreads();
-      const int steps = (n + kThreads - 1) / kThreads;
-      for (int st = 0; st < steps; ++st) {
-        const int t = st * kThreads + tid;
-        int b = -1;
-        uint32_t key = 0;
-        if (t < n) {
-          b = S.bucket_of_role[roles[t]];
-          key = keys[t];
-          if (b >= 0 && (S.mode[b] != 2 || (key & hi_mask) != S.prefix[b])) b = -1;
-        }
-        const int digit = (key >> shift) & 255;
-        const int tag = (b < 0) ? -1 : (b << 8) | digit;
-        const unsigned peers = __match_any_sync(0xffffffffu, tag);
-        if (tag >= 0 && (__ffs(peers) - 1) == lane)
-          atomicAdd(&S.hist[b][digit], __popc(peers));
+  // A NaN score (or +inf and -inf in one group): redo the keys one token at a
+  // time, a window holding a NaN giving the lowest key.
+  if (S.nan_hint) {
+    const int hw = a.pool_k / 2;
+    uint32_t* kw = reinterpret_cast<uint32_t*>(keys4);
+    bool seen = false;
+    for (int t = tid; t < n; t += NT) {
+      const int lo = max(0, t - hw), hi = min(n - 1, t + hw);
+      float m = __ldg(v.sp + lo);
+      bool nan_w = isnan(m);
+      for (int x = lo + 1; x <= hi; ++x) {
+        const float f = __ldg(v.sp + x);
+        nan_w |= isnan(f);
+        m = fmaxf(m, f);
       }
-      __syncthreads();
-      if (warp < kR && S.mode[warp] == 2) {
-        const int b = warp;
-        // lane handles digits [lane*8, lane*8+8); suffix sums from the top
-        int c[8];
-        int mine = 0;
+      seen |= nan_w;
+      kw[t + off] = nan_w ? 0u : ordered_key(m);
+    }
+    if (__any_sync(0xffffffffu, seen) && lane == 0) S.nan_seen = 1;
+  }
+
+  // ---- quotas and the role -> code table
+  if (warp == 0) quotas_warp(a, lane, K_s, S);
+  __syncthreads();
+  for (int x = tid; x < 256; x += NT) {
+    uint32_t code = kCodeDrop;
+    if (x < a.n_roles && !((a.ban_mask >> x) & 1u)) {
+      const int b = (a.policy == ROLEKV_POLICY_GLOBAL) ? 0 : x;
+      code = S.mode[b] == 2 ? static_cast<uint32_t>(b) : (S.mode[b] == 1 ? kCodeKeep : kCodeDrop);
+    }
+    S.code_of_role[x] = static_cast<int32_t>(code);
+  }
+  const bool any_thr = S.any_threshold != 0;
+  if (tid == 0 && (S.nan_hint || ((S.top_and ^ S.top_or) & 0x80000000u))) S.general = 1;
+  __syncthreads();
+
+  // ---- first digit per bucket
+  if (any_thr && !S.general) {
+    if (warp < kR && S.mode[warp] == 2) descend_first(a, S, hist16, warp, lane, nb);
+    __syncthreads();
+    if (tid == 0) {
+      int total = 0;
+      for (int b = 0; b < kR; ++b) total += S.mode[b] == 2 ? S.cand[b] : 0;
+      if (total > list_cap) S.general = 1;
+    }
+    __syncthreads();
+  }
+
+  const int sh0 = 31 - nb;
+  if (!S.general) {
+    // ---- pass 2: decide every token outside its bucket's threshold digit,
+    // list the rest
+    for (int i = 0; i < iters; ++i) {
+      const int g = i * NT + tid;
+      uint32_t m4 = 0, c4 = 0;
+      uint32_t ent[4] = {0u, 0u, 0u, 0u};
+      if (g < ngroups) {
+        const uint4 kv = keys4[g];
+        const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
+        const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          c[i] = S.hist[b][lane * 8 + i];
-          mine += c[i];
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t code = static_cast<uint32_t>(S.code_of_role[(rw >> (8 * j)) & 0xFFu]);
+          bool keep = code == kCodeKeep;
+          if (code < static_cast<uint32_t>(kR)) {
+            const uint32_t hb = kk[j] >> sh0, pb = S.prefix[code] >> sh0;
+            keep = hb > pb;
+            if (hb == pb) {
+              c4 |= 1u << j;
+              ent[j] = (code << 16) | static_cast<uint32_t>(4 * g + j);
+            }
+          }
+          m4 |= static_cast<uint32_t>(keep) << j;
         }
-        // above = tokens whose digit falls in a higher lane's range
-        int incl = mine;
+      }
+      store_bits(bits, g, nwords, lane, m4);
+      const int nc = __popc(c4);
+      if (__any_sync(0xffffffffu, nc != 0)) {
+        int incl = nc;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
-          const int v = __shfl_down_sync(0xffffffffu, incl, o);
-          if (lane + o < 32) incl += v;
+          const int t = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += t;
         }
-        const int above = incl - mine;
-        const int need = static_cast<int>(S.need[b]);
-        // the digit where the count of larger-or-equal keys first reaches need
-        int found_digit = -1, gt_before = 0;
-        if (above < need && above + mine >= need) {
-          int acc = above;
-          for (int i = 7; i >= 0; --i) {
-            if (acc + c[i] >= need) {
-              found_digit = lane * 8 + i;
-              gt_before = acc;
-              break;
-            }
-            acc += c[i];
+        int base = 0;
+        if (lane == 31) base = atomicAdd(&S.list_n, incl);
+        base = __shfl_sync(0xffffffffu, base, 31);
+        int pos = base + incl - nc;
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          if ((c4 >> j) & 1u) {
+            if (pos < list_cap) list[pos] = ent[j];
+            ++pos;
           }
-        }
-        const unsigned who = __ballot_sync(0xffffffffu, found_digit >= 0);
-        const int src = who ? __ffs(who) - 1 : 0;
-        const int fd = __shfl_sync(0xffffffffu, found_digit, src);
-        const int gb = __shfl_sync(0xffffffffu, gt_before, src);
-        if (lane == 0 && who != 0) {
-          S.prefix[b] |= static_cast<uint32_t>(fd) << shift;
-          S.need[b] = static_cast<uint32_t>(need - gb);
-        }
       }
+    }
+    __syncthreads();
+    if (S.list_n > list_cap) {
+      if (tid == 0) S.general = 1;   // (cannot happen: the counts bound the list)
       __syncthreads();
     }
   }
 
-  // ---- tie ranks in index order and the kept set.  Warp w owns the token
-  // range [w*seg, (w+1)*seg).
-  const int seg = ((n + kWarps - 1) / kWarps + 31) & ~31;
-  const int t_begin = warp * seg;
-  const int t_end = min(n, t_begin + seg);
-  const unsigned lt_mask = (1u << lane) - 1u;
-  // pass A: ties per bucket in this warp's range
-  {
-    int tie_cnt[kR];
-#pragma unroll
-    for (int r = 0; r < kR; ++r) tie_cnt[r] = 0;
-    for (int t0 = t_begin; t0 < t_end; t0 += 32) {
-      const int t = t0 + lane;
-      int b = -1;
-      if (t < t_end) {
-        b = S.bucket_of_role[roles[t]];
-        if (b >= 0 && !(S.mode[b] == 2 && keys[t] == S.prefix[b])) b = -1;
+  if (!S.general) {
+    if (any_thr) {
+      // ---- remaining bits over the candidate list
+      const int m = S.list_n;
+      for (int lo = sh0; lo > 0;) {
+        const int d = lo < 8 ? lo : 8;
+        const int shift = lo - d;
+        for (int e = tid; e < m; e += NT) {
+          const uint32_t ent = list[e];
+          const uint32_t c = ent >> 16;
+          const uint32_t key = keys[ent & 0xFFFFu];
+          if ((key >> lo) == (S.prefix[c] >> lo))
+            atomicAdd(&S.hist[c][(key >> shift) & ((1u << d) - 1u)], 1);
+        }
+        __syncthreads();
+        if (warp < kR && S.mode[warp] == 2) descend(S, warp, lane, shift);
+        __syncthreads();
+        lo = shift;
       }
-#pragma unroll
-      for (int r = 0; r < kR; ++r) tie_cnt[r] += __popc(__ballot_sync(0xffffffffu, b == r));
-    }
-    if (lane < kR) {
-      int v = 0;
-#pragma unroll
-      for (int r = 0; r < kR; ++r) v = (lane == r) ? tie_cnt[r] : v;
-      S.warp_cnt[warp][lane] = v;
-    }
-  }
-  __syncthreads();
-  if (tid < kR) {   // exclusive scan over warps, bucket `tid`
-    int run = 0;
-    for (int w = 0; w < kWarps; ++w) {
-      const int v = S.warp_cnt[w][tid];
-      S.warp_cnt[w][tid] = run;
-      run += v;
-    }
-  }
-  __syncthreads();
-  // pass B: decide, record bits, count per warp and per role
-  {
-    int tie_run[kR];
-#pragma unroll
-    for (int r = 0; r < kR; ++r) tie_run[r] = S.warp_cnt[warp][r];
-    int kept_here = 0;
-    int role_kept[kR];
-#pragma unroll
-    for (int r = 0; r < kR; ++r) role_kept[r] = 0;
-    for (int t0 = t_begin; t0 < t_end; t0 += 32) {
-      const int t = t0 + lane;
-      bool keep = false;
-      int b = -1, tie_b = -1, role = 0;
-      if (t < t_end) {
-        role = roles[t];
-        b = S.bucket_of_role[role];
-        if (b >= 0) {
-          const int md = S.mode[b];
-          if (md == 1) {
-            keep = true;
-          } else if (md == 2) {
-            const uint32_t k = keys[t];
-            if (k > S.prefix[b]) keep = true;
-            else if (k == S.prefix[b]) tie_b = b;
-          }
+      // kept candidates join the bits; ties of partial buckets are gathered
+      const uint32_t partial = S.partial_ties;
+      for (int e = tid; e < m; e += NT) {
+        const uint32_t ent = list[e];
+        const uint32_t c = ent >> 16, slot = ent & 0xFFFFu;
+        const uint32_t key = keys[slot];
+        if (key >= S.thr[c]) {
+          atomicOr(&bits[slot >> 5], 1u << (slot & 31u));
+        } else if (((partial >> c) & 1u) && key == S.prefix[c]) {
+          const int t = atomicAdd(&S.tie_n, 1);
+          if (t < kTieCap) S.ties[t] = ent;
         }
       }
+      __syncthreads();
+      const int nt = S.tie_n;
+      if (partial != 0 && nt <= kTieCap) {
+        // index-order rank among the bucket's ties
+        for (int t = tid; t < nt; t += NT) {
+          const uint32_t ent = S.ties[t];
+          const uint32_t c = ent >> 16, slot = ent & 0xFFFFu;
+          int rank = 0;
+          for (int x = 0; x < nt; ++x) {
+            const uint32_t o = S.ties[x];
+            rank += ((o >> 16) == c && (o & 0xFFFFu) < slot);
+          }
+          if (rank < S.need[c]) atomicOr(&bits[slot >> 5], 1u << (slot & 31u));
+        }
+        __syncthreads();
+      } else if (partial != 0) {
+        if (tid == 0) S.general = 2;   // too many ties: rank them over all slots
+        __syncthreads();
+      }
+    }
+  } else {
+    // ---- general path: four 8-bit rounds over every slot, from the top
+    // (the first-digit step may have run before the list overflowed)
+    if (tid < kR) {
+      S.prefix[tid] = 0;
+      S.need[tid] = S.quota[tid];
+    }
+    __syncthreads();
+    for (int round = 0; round < (any_thr ? 4 : 0); ++round) {
+      const int shift = 24 - 8 * round;
+      for (int i = 0; i < iters; ++i) {
+        const int g = i * NT + tid;
+        if (g >= ngroups) break;
+        const uint4 kv = keys4[g];
+        const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
+        const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t c = static_cast<uint32_t>(S.code_of_role[(rw >> (8 * j)) & 0xFFu]);
+          if (c >= static_cast<uint32_t>(kR)) continue;
+          if (round > 0 && (kk[j] >> (shift + 8)) != (S.prefix[c] >> (shift + 8))) continue;
+          atomicAdd(&S.hist[c][(kk[j] >> shift) & 0xFFu], 1);
+        }
+      }
+      __syncthreads();
+      if (warp < kR && S.mode[warp] == 2) descend(S, warp, lane, shift);
+      __syncthreads();
+    }
+    for (int i = 0; i < iters; ++i) {
+      const int g = i * NT + tid;
+      uint32_t m4 = 0;
+      if (g < ngroups) {
+        const uint4 kv = keys4[g];
+        const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
+        const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t c = static_cast<uint32_t>(S.code_of_role[(rw >> (8 * j)) & 0xFFu]);
+          const bool keep = (c < static_cast<uint32_t>(kR)) ? (kk[j] >= S.thr[c]) : (c == kCodeKeep);
+          m4 |= static_cast<uint32_t>(keep) << j;
+        }
+      }
+      store_bits(bits, g, nwords, lane, m4);
+    }
+    __syncthreads();
+  }
+
+  // Ties beyond the shared-memory list (general path, or too many ties): the
+  // first need[b] keys equal to the threshold, in index order, over all slots.
+  if (S.general) {
+    for (uint32_t pend = S.partial_ties; pend != 0; pend &= pend - 1) {
+      const int b = __ffs(pend) - 1;
+      const uint32_t P = S.prefix[b];
+      const int need = S.need[b];
+      auto tie_mask = [&](int q) {
+        uint32_t mk = 0;
+#pragma unroll
+        for (int gg = 0; gg < 8; ++gg) {
+          const int g = 8 * q + gg;
+          if (g >= ngroups) break;
+          const uint4 kv = keys4[g];
+          const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
+          const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            if (S.code_of_role[(rw >> (8 * j)) & 0xFFu] == b && kk[j] == P) mk |= 1u << (4 * gg + j);
+        }
+        return mk;
+      };
+      scan_words<NT>(nwords, tie_mask, [&](int q, uint32_t mk, int rank) {
+        uint32_t keepm = 0;
+        while (mk != 0 && rank < need) {
+          const uint32_t low = mk & (0u - mk);
+          keepm |= low;
+          mk ^= low;
+          ++rank;
+        }
+        if (keepm) bits[q] |= keepm;
+      }, S.warp_tot);
+    }
+  }
+
+  // ---- kept positions in ascending order
+  int32_t* dst = a.keep_idx + S.keep_off;
+  const bool count_roles = a.kept_per_role != nullptr && a.policy == ROLEKV_POLICY_GLOBAL;
+  uint64_t kr = 0;
+  const int total = scan_words<NT>(nwords, [&](int q) { return bits[q]; }, [&](int q, uint32_t m, int pos) {
+    while (m != 0) {
+      const int t = q * 32 + (__ffs(m) - 1) - off;
+      m &= m - 1;
+      dst[pos++] = t;
+      if (count_roles) kr += shl64(1ull, 8u * __ldg(v.rp + t));
+    }
+  }, S.warp_tot);
+  for (int64_t j = total + tid; j < K_s; j += NT) dst[j] = -1;
+
+  if (a.keep_mask != nullptr) {
+    uint8_t* mp = a.keep_mask + sbase;
+    const bool mvec = ((reinterpret_cast<uintptr_t>(mp) - static_cast<uintptr_t>(off)) & 3u) == 0;
+    for (int g = tid; g < ngroups; g += NT) {
+      const uint32_t m4 = (bits[g >> 3] >> (4 * (g & 7))) & 15u;
+      const int s0 = 4 * g - off;
+      if (mvec && s0 >= 0 && s0 + 4 <= n) {
+        const uint32_t w = (m4 & 1u) | ((m4 >> 1) & 1u) << 8 | ((m4 >> 2) & 1u) << 16 | ((m4 >> 3) & 1u) << 24;
+        *reinterpret_cast<uint32_t*>(mp + s0) = w;
+      } else {
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          if (s0 + j >= 0 && s0 + j < n) mp[s0 + j] = static_cast<uint8_t>((m4 >> j) & 1u);
+      }
+    }
+  }
+
+  if (a.kept_per_role != nullptr) {
+    if (count_roles) {
 #pragma unroll
       for (int r = 0; r < kR; ++r) {
-        const unsigned m = __ballot_sync(0xffffffffu, tie_b == r);
-        if (tie_b == r) keep = (tie_run[r] + __popc(m & lt_mask)) < static_cast<int>(S.need[r]);
-        tie_run[r] += __popc(m);
+        const int c = warp_sum(static_cast<int>((kr >> (8 * r)) & 0xFFu));
+        if (lane == 0 && c) atomicAdd(&S.kept_role[r], c);
       }
-      const unsigned km = __ballot_sync(0xffffffffu, keep);
-      if (lane == 0 && t0 < t_end) {
-        // bits of tokens t0 .. t0+31 (t0 is a multiple of 32)
-        keptbits[t0 >> 5] = km;
-      }
-      kept_here += __popc(km);
-      if (keep) {
-#pragma unroll
-        for (int r = 0; r < kR; ++r) role_kept[r] += (role == r);
-      }
-      if (a.keep_mask != nullptr && t < t_end) a.keep_mask[sbase + t] = keep ? 1 : 0;
+      __syncthreads();
     }
-    if (lane == 0) S.warp_kept[warp] = kept_here;
-    if (a.kept_per_role != nullptr) {
-#pragma unroll
-      for (int r = 0; r < kR; ++r) {
-        const int v = warp_sum(role_kept[r]);
-        if (lane == 0 && v) atomicAdd(&S.kept_role[r], v);
-      }
-    }
+    if (tid < a.n_roles)
+      a.kept_per_role[static_cast<int64_t>(u) * a.n_roles + tid] =
+          count_roles ? S.kept_role[tid] : S.quota[tid];
   }
-  __syncthreads();
-  if (tid == 0) {
-    int run = 0;
-    for (int w = 0; w < kWarps; ++w) {
-      const int v = S.warp_kept[w];
-      S.warp_kept[w] = run;
-      run += v;
-    }
-    S.warp_cnt[0][0] = run;   // total kept (the scan above is no longer needed)
-  }
-  __syncthreads();
-  // pass C: write kept positions in ascending order
-  {
-    int out = S.warp_kept[warp];
-    int32_t* dst = a.keep_idx + S.keep_off;
-    for (int t0 = t_begin; t0 < t_end; t0 += 32) {
-      const unsigned km = keptbits[t0 >> 5];
-      if ((km >> lane) & 1u) dst[out + __popc(km & lt_mask)] = t0 + lane;
-      out += __popc(km);
-    }
-    const int total = S.warp_cnt[0][0];
-    for (int64_t j = total + tid; j < K_s; j += kThreads) dst[j] = -1;
-  }
-  if (a.kept_per_role != nullptr && tid < a.n_roles)
-    a.kept_per_role[static_cast<int64_t>(u) * a.n_roles + tid] = S.kept_role[tid];
-  if (tid == 0 && S.nonfinite && a.status != nullptr) atomicOr(a.status, ROLEKV_STATUS_NONFINITE);
+  if (tid == 0 && S.nan_seen && a.status != nullptr) atomicOr(a.status, ROLEKV_STATUS_NONFINITE);
+}
+
+template <int NT>
+cudaError_t launch_select_nt(const SelectArgs& a, size_t smem, cudaStream_t stream) {
+  cudaError_t e = cudaFuncSetAttribute(select_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  select_kernel<NT><<<a.n_units, NT, smem, stream>>>(a);
+  return cudaGetLastError();
 }
 
 }  // namespace
 
 size_t select_smem_bytes(int n_max) {
-  const size_t keys = static_cast<size_t>(n_max) * 4;
-  const size_t roles = (static_cast<size_t>(n_max) + 15) & ~static_cast<size_t>(15);
-  const size_t bits = ((static_cast<size_t>(n_max) + 31) / 32 + 32) * 4;
-  return keys + roles + bits;
+  const size_t groups = static_cast<size_t>(select_groups(n_max));
+  return groups * 16 + groups / 8 * 4 + region_bytes(n_max);
 }
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream) {
   if (a.n_units == 0) return cudaSuccess;
   const size_t smem = select_smem_bytes(a.n_max);
-  cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
-  if (e != cudaSuccess) return e;
-  select_kernel<<<a.n_units, kThreads, smem, stream>>>(a);
-  return cudaGetLastError();
+  // CTA size follows the row length so that short rows still fill the SM
+  // with several CTAs (shared memory is sized by the longest row).
+  if (a.n_max > 16384) return launch_select_nt<1024>(a, smem, stream);
+  if (a.n_max > 8192) return launch_select_nt<512>(a, smem, stream);
+  return launch_select_nt<256>(a, smem, stream);
 }
 
 }  // namespace rolekv

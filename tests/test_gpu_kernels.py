@@ -137,6 +137,8 @@ SELECT_CASES = [
     ("global_no_key", _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=4000), 0.30, 0.0, 1, 1 << I.ROLE_KEY, 1),
     ("global_plain", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=4000), 0.20, 0.0, 1, 0, 5),
     ("varlen", _w("ragged", L=2, b=4, Hq=8, Hkv=2, n=3000, seqlens=(3000, 0, 5, 1200)), 0.10, 0.0, 0, 0, 7),
+    ("mid_n", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=12001), 0.10, 0.02, 0, 0, 7),
+    ("mid_n_global_pool15", _w("llama8b", L=1, b=1, Hq=4, Hkv=1, n=9999), 0.10, 0.0, 1, 0, 15),
     ("max_n", _w("long", L=1, b=1, Hq=4, Hkv=1, n=R.SELECT_MAX_N), 0.10, 0.0, 0, 0, 7),
 ]
 
@@ -182,6 +184,40 @@ def test_role_alloc_select_bit_exact(case):
         assert np.array_equal(m, expect), f"{name} unit {u} mask"
         if akey == 0.0 and policy == 0:
             assert per[I.ROLE_KEY] == 0
+
+
+@pytest.mark.parametrize("pool_k", [1, 7])
+def test_select_nan_scores_flagged_and_lowest(pool_k):
+    """A NaN score sets STATUS_NONFINITE; every pooled window holding a NaN
+    ranks below every other token (kept last, ties in index order)."""
+    w = _w("llama8b", L=1, b=2, Hq=4, Hkv=1, n=3001)
+    roles_np = I.workload_roles(w, 4)
+    batch = lib_batch(w, DEV)
+    g = torch.Generator().manual_seed(11)
+    sc = torch.rand(batch.score_shape(), generator=g)
+    flat = sc.view(-1)
+    flat[torch.randint(0, flat.numel(), (40,), generator=g)] = float("nan")
+    B = 0.60
+    keep = torch.empty(batch.kept_shape(B), dtype=torch.int32, device=DEV)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    R.role_alloc_select(batch, sc.to(DEV), torch.as_tensor(roles_np, device=DEV),
+                        R.select_params(B, I.PAPER_ALPHA, 0.0, I.ROLE_KEY), keep, pool_k=pool_k,
+                        status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) & R.STATUS_NONFINITE
+    ob = oracle_batch(w)
+    sc_np = sc.numpy()
+    unit_scores = {}
+    for u in range(ob.n_units):
+        x = ob.score_view(sc_np, u).astype(np.float64)
+        hw = pool_k // 2
+        nan_win = np.array([np.isnan(x[max(0, t - hw):t + hw + 1]).any() for t in range(x.size)])
+        pooled = O.maxpool1d(np.where(np.isnan(x), -np.inf, x), pool_k)
+        unit_scores[u] = np.where(nan_win, -np.inf, pooled)
+    ref = O.select_batch(ob, unit_scores, roles_np, I.N_ROLES, I.PAPER_ALPHA, I.ROLE_KEY, 0.0, B)
+    got = keep.cpu().numpy().reshape(ob.n_units, -1)
+    for u, (idx, _) in ref.items():
+        assert np.array_equal(got[u], idx), f"unit {u}"
 
 
 def test_select_infeasible_budget_pads():

@@ -12,9 +12,10 @@
 //
 // The threshold of each bucket is found by a radix descent over the keys'
 // bits, most significant first:
-//   pass 1  load, pool, key; role counts and, per role, a histogram of the
-//           key's bits 30..31-NB (the top bit is shared by every key when all
-//           scores have one sign): exponent and leading mantissa bits.
+//   pass 1  load, pool, key; per role, a histogram of the key's bits
+//           30..31-NB (the top bit is shared by every key when all scores
+//           have one sign): exponent and leading mantissa bits.  The role
+//           counts are the histograms' sums.
 //   quotas  one warp, lane r for role r (water-filling, largest remainders).
 //   first digit from the pass-1 histograms, per bucket.
 //   pass 2  every token is decided (kept / dropped) unless its first digit is
@@ -98,6 +99,7 @@ struct SelShared {
   int32_t mode[kR];        // 0 none kept, 1 all kept, 2 threshold
   int32_t cand[kR];        // candidates after the first digit
   int32_t code_of_role[256];
+  int32_t first_of_role[256];  // pass 2: keep iff first digit > it, candidate iff ==
   int32_t hist[kR][256];
   int32_t warp_tot[32];
   int32_t kept_role[kR];
@@ -148,8 +150,8 @@ struct UnitView {
 // Pass 1 for a pool half-width HW known at compile time.
 template <int HW, int NT>
 __device__ __forceinline__ void pass1(const UnitView& v, int n_roles, int nb, uint4* keys4,
-                                      uint32_t* hist16, uint64_t& rc, bool& nan_hint,
-                                      uint32_t& top_and, uint32_t& top_or) {
+                                      uint32_t* hist16, bool& nan_hint, uint32_t& top_and,
+                                      uint32_t& top_or) {
   constexpr int NB = (HW + 3) / 4;   // neighbour groups on each side
   const int sh0 = 31 - nb;
   const uint32_t bmask = (1u << nb) - 1u;
@@ -185,7 +187,6 @@ __device__ __forceinline__ void pass1(const UnitView& v, int n_roles, int nb, ui
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       const uint32_t r = (rw >> (8 * j)) & 0xFFu;
-      rc += shl64(1ull, 8u * r);
       if (r < static_cast<uint32_t>(n_roles)) {
         top_and &= k[j];
         top_or |= k[j];
@@ -199,25 +200,34 @@ __device__ __forceinline__ void pass1(const UnitView& v, int n_roles, int nb, ui
 // Quotas of one sequence by warp 0, lane r for role r: water-filling of the
 // weights over the role counts, then the integer remainders to the largest
 // fractional parts (ties to the lower role), the arithmetic stated in rolekv.h.
+__device__ __forceinline__ int64_t sum8(int64_t v) {
+  v += __shfl_xor_sync(0xffffffffu, v, 1);
+  v += __shfl_xor_sync(0xffffffffu, v, 2);
+  v += __shfl_xor_sync(0xffffffffu, v, 4);
+  return v;
+}
+
 __device__ void quotas_warp(const SelectArgs& a, int lane, int64_t K_full, SelShared& S) {
-  const int r = lane;
+  // every group of 8 lanes holds the 8 roles, so sums over a group are the
+  // totals and all lanes take the same branches
+  const int r = lane & (kR - 1);
   const bool valid = r < a.n_roles;
   const bool banned = valid && ((a.ban_mask >> r) & 1u);
   const int64_t cnt = valid ? S.count[r] : 0;
   const int64_t alpha = r < kR ? a.alpha_fx[r] : 0;
   int64_t q = 0, bsize = 0;
   if (a.policy == ROLEKV_POLICY_GLOBAL) {
-    const int64_t elig = warp_sum64((valid && !banned) ? cnt : 0);
+    const int64_t elig = sum8((valid && !banned) ? cnt : 0);
     if (r == 0) {
       q = K_full < elig ? K_full : elig;
       bsize = elig;
     }
   } else {
     bool live = valid && alpha > 0 && cnt > 0;
-    const int64_t elig = warp_sum64(live ? cnt : 0);
+    const int64_t elig = sum8(live ? cnt : 0);
     int64_t left = K_full < elig ? K_full : elig;
     for (int it = 0; it <= kR; ++it) {
-      const int64_t A = warp_sum64(live ? alpha : 0);
+      const int64_t A = sum8(live ? alpha : 0);
       if (A == 0) break;
       const bool sat = live && alpha * left >= cnt * A;
       if (!__any_sync(0xffffffffu, sat)) break;
@@ -225,15 +235,15 @@ __device__ void quotas_warp(const SelectArgs& a, int lane, int64_t K_full, SelSh
         q = cnt;
         live = false;
       }
-      left -= warp_sum64(sat ? cnt : 0);
+      left -= sum8(sat ? cnt : 0);
     }
-    const int64_t A = warp_sum64(live ? alpha : 0);
+    const int64_t A = sum8(live ? alpha : 0);
     int64_t rem = -1;
     if (live && A != 0) {
       q = alpha * left / A;
       rem = alpha * left % A;
     }
-    const int64_t extra = left - warp_sum64(live ? q : 0);
+    const int64_t extra = left - sum8(live ? q : 0);
     int rank = 0;
 #pragma unroll
     for (int x = 0; x < kR; ++x) {
@@ -245,7 +255,7 @@ __device__ void quotas_warp(const SelectArgs& a, int lane, int64_t K_full, SelSh
     bsize = cnt;
   }
   int mode = 0;
-  if (r < kR) {
+  if (lane < kR) {
     mode = (q <= 0) ? 0 : (q >= bsize ? 1 : 2);
     S.quota[r] = static_cast<int32_t>(q);
     S.mode[r] = mode;
@@ -318,25 +328,42 @@ __device__ void descend(SelShared& S, int b, int lane, int shift) {
 
 // First digit (bits 30..31-nb, the shared top bit above them) of bucket b from
 // the per-role 16-bit histograms of pass 1; the bucket's histogram is the sum
-// over its roles.
+// over its roles.  Lane L owns a contiguous range of bins: the lanes' totals
+// (read in a rotated order, so that the lanes hit different banks) locate the
+// lane holding the threshold, then the warp splits that lane's words.
+template <int NB>
 __device__ void descend_first(const SelectArgs& a, SelShared& S, const uint32_t* hist16, int b,
-                              int lane, int nb) {
-  const int bpl = 1 << (nb - 5);   // bins per lane
-  const int wpr = 1 << (nb - 1);   // words per role
+                              int lane) {
+  constexpr int nb = NB;
+  constexpr int wpl = 1 << (nb - 6);   // histogram words (two bins each) per lane
+  constexpr int wpr = 1 << (nb - 1);   // words per role
   const uint32_t roles = (a.policy == ROLEKV_POLICY_GLOBAL)
                              ? (((1u << a.n_roles) - 1u) & ~a.ban_mask)
                              : (1u << b);
-  auto count = [&](int bin) {
-    int s = 0;
-    for (uint32_t m = roles; m != 0; m &= m - 1) {
-      const int r = __ffs(m) - 1;
-      s += static_cast<int>((hist16[r * wpr + (bin >> 1)] >> (16 * (bin & 1))) & 0xFFFFu);
-    }
-    return s;
+  // counts of bins 2w (low half) and 2w+1 (high half), summed over the roles;
+  // a bin holds at most n < 65536 tokens, so the halves never carry
+  const bool single = (roles & (roles - 1)) == 0;
+  const uint32_t* h0 = hist16 + (__ffs(roles) - 1) * wpr;
+  auto word = [&](int w) {
+    if (single) return h0[w];
+    uint32_t x = 0;
+    for (uint32_t m = roles; m != 0; m &= m - 1) x += hist16[(__ffs(m) - 1) * wpr + w];
+    return x;
   };
   int mine = 0;
-  for (int i = 0; i < bpl; ++i) mine += count(lane * bpl + i);
-  int incl = mine;
+  if (single) {
+#pragma unroll
+    for (int i = 0; i < wpl; ++i) {
+      const uint32_t x = h0[lane * wpl + ((i + lane) & (wpl - 1))];
+      mine += static_cast<int>((x & 0xFFFFu) + (x >> 16));
+    }
+  } else {
+    for (int i = 0; i < wpl; ++i) {
+      const uint32_t x = word(lane * wpl + ((i + lane) & (wpl - 1)));
+      mine += static_cast<int>((x & 0xFFFFu) + (x >> 16));
+    }
+  }
+  int incl = mine;   // tokens in this lane's bins or above
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
     const int v = __shfl_down_sync(0xffffffffu, incl, o);
@@ -344,34 +371,45 @@ __device__ void descend_first(const SelectArgs& a, SelShared& S, const uint32_t*
   }
   const int above = incl - mine;
   const int need = S.need[b];
-  int found = -1, gt_before = 0, at_digit = 0;
-  if (above < need && above + mine >= need) {
-    int acc = above;
-    for (int i = bpl - 1; i >= 0; --i) {
-      const int ci = count(lane * bpl + i);
-      if (acc + ci >= need) {
-        found = lane * bpl + i;
-        gt_before = acc;
-        at_digit = ci;
-        break;
-      }
-      acc += ci;
-    }
+  const unsigned who = __ballot_sync(0xffffffffu, above < need && above + mine >= need);
+  if (who == 0) {
+    if (lane == 0) S.general = 1;   // counts disagree with the quota: let the full path decide
+    return;
   }
-  const unsigned who = __ballot_sync(0xffffffffu, found >= 0);
-  const int src = who ? __ffs(who) - 1 : 0;
-  const int fd = __shfl_sync(0xffffffffu, found, src);
-  const int gb = __shfl_sync(0xffffffffu, gt_before, src);
-  const int ad = __shfl_sync(0xffffffffu, at_digit, src);
-  if (lane == 0) {
-    if (who == 0) {
-      S.general = 1;   // counts disagree with the quota: let the full path decide
+  const int F = __ffs(who) - 1;
+  const int aboveF = __shfl_sync(0xffffffffu, above, F);
+  const int needF = need - aboveF;
+  const uint32_t x = lane < wpl ? word(F * wpl + lane) : 0u;
+  const int lo = static_cast<int>(x & 0xFFFFu), hi = static_cast<int>(x >> 16);
+  const int pair = lo + hi;
+  int incl2 = pair;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int v = __shfl_down_sync(0xffffffffu, incl2, o);
+    if (lane + o < 32) incl2 += v;
+  }
+  const int above2 = incl2 - pair;
+  const unsigned who2 = __ballot_sync(0xffffffffu, above2 < needF && above2 + pair >= needF);
+  if (who2 == 0) {
+    if (lane == 0) S.general = 1;
+    return;
+  }
+  if (lane == __ffs(who2) - 1) {
+    const int w = F * wpl + lane;
+    int fd, gb, ad;
+    if (above2 + hi >= needF) {
+      fd = 2 * w + 1;
+      gb = aboveF + above2;
+      ad = hi;
     } else {
-      const int sh0 = 31 - nb;
-      S.prefix[b] = (S.top_and & 0x80000000u) | (static_cast<uint32_t>(fd) << sh0);
-      S.need[b] = need - gb;
-      S.cand[b] = ad;
+      fd = 2 * w;
+      gb = aboveF + above2 + hi;
+      ad = lo;
     }
+    const int sh0 = 31 - nb;
+    S.prefix[b] = (S.top_and & 0x80000000u) | (static_cast<uint32_t>(fd) << sh0);
+    S.need[b] = need - gb;
+    S.cand[b] = ad;
   }
 }
 
@@ -508,25 +546,19 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
     }
   }
 
-  // ---- pass 1: load, pool, key, role counts, first-digit histograms
+  // ---- pass 1: load, pool, key, first-digit histograms
   {
-    uint64_t rc = 0;
     bool nan_hint = false;
     uint32_t tand = 0xFFFFFFFFu, tor = 0u;
     switch (a.pool_k >> 1) {
-      case 0: pass1<0, NT>(v, a.n_roles, nb, keys4, hist16, rc, nan_hint, tand, tor); break;
-      case 1: pass1<1, NT>(v, a.n_roles, nb, keys4, hist16, rc, nan_hint, tand, tor); break;
-      case 2: pass1<2, NT>(v, a.n_roles, nb, keys4, hist16, rc, nan_hint, tand, tor); break;
-      case 3: pass1<3, NT>(v, a.n_roles, nb, keys4, hist16, rc, nan_hint, tand, tor); break;
-      case 4: pass1<4, NT>(v, a.n_roles, nb, keys4, hist16, rc, nan_hint, tand, tor); break;
-      case 5: pass1<5, NT>(v, a.n_roles, nb, keys4, hist16, rc, nan_hint, tand, tor); break;
-      case 6: pass1<6, NT>(v, a.n_roles, nb, keys4, hist16, rc, nan_hint, tand, tor); break;
-      default: pass1<7, NT>(v, a.n_roles, nb, keys4, hist16, rc, nan_hint, tand, tor); break;
-    }
-#pragma unroll
-    for (int r = 0; r < kR; ++r) {
-      const int c = warp_sum(static_cast<int>((rc >> (8 * r)) & 0xFFu));
-      if (lane == 0 && c) atomicAdd(&S.count[r], c);
+      case 0: pass1<0, NT>(v, a.n_roles, nb, keys4, hist16, nan_hint, tand, tor); break;
+      case 1: pass1<1, NT>(v, a.n_roles, nb, keys4, hist16, nan_hint, tand, tor); break;
+      case 2: pass1<2, NT>(v, a.n_roles, nb, keys4, hist16, nan_hint, tand, tor); break;
+      case 3: pass1<3, NT>(v, a.n_roles, nb, keys4, hist16, nan_hint, tand, tor); break;
+      case 4: pass1<4, NT>(v, a.n_roles, nb, keys4, hist16, nan_hint, tand, tor); break;
+      case 5: pass1<5, NT>(v, a.n_roles, nb, keys4, hist16, nan_hint, tand, tor); break;
+      case 6: pass1<6, NT>(v, a.n_roles, nb, keys4, hist16, nan_hint, tand, tor); break;
+      default: pass1<7, NT>(v, a.n_roles, nb, keys4, hist16, nan_hint, tand, tor); break;
     }
     tand = __reduce_and_sync(0xffffffffu, tand);
     tor = __reduce_or_sync(0xffffffffu, tor);
@@ -538,6 +570,17 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
     }
   }
   __syncthreads();
+
+  // Role counts: the sums of the roles' histograms (a warp's 32 words belong
+  // to one role).
+  {
+    const int wpr = 1 << (nb - 1);
+    for (int x0 = warp * 32; x0 < a.n_roles * wpr; x0 += NT) {
+      const uint32_t w = hist16[x0 + lane];
+      const int c = warp_sum(static_cast<int>((w & 0xFFFFu) + (w >> 16)));
+      if (lane == 0 && c) atomicAdd(&S.count[x0 >> (nb - 1)], c);
+    }
+  }
 
   // A NaN score (or +inf and -inf in one group): redo the keys one token at a
   // time, a window holding a NaN giving the lowest key.
@@ -559,6 +602,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
     }
     if (__any_sync(0xffffffffu, seen) && lane == 0) S.nan_seen = 1;
   }
+  __syncthreads();
 
   // ---- quotas and the role -> code table
   if (warp == 0) quotas_warp(a, lane, K_s, S);
@@ -577,7 +621,12 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
 
   // ---- first digit per bucket
   if (any_thr && !S.general) {
-    if (warp < kR && S.mode[warp] == 2) descend_first(a, S, hist16, warp, lane, nb);
+    if (warp < kR && S.mode[warp] == 2) {
+      if (nb == 11)
+        descend_first<11>(a, S, hist16, warp, lane);
+      else
+        descend_first<10>(a, S, hist16, warp, lane);
+    }
     __syncthreads();
     if (tid == 0) {
       int total = 0;
@@ -589,44 +638,56 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
 
   const int sh0 = 31 - nb;
   if (!S.general) {
+    for (int x = tid; x < 256; x += NT) {
+      const uint32_t code = static_cast<uint32_t>(S.code_of_role[x]);
+      S.first_of_role[x] = code == kCodeKeep                  ? -1
+                           : code < static_cast<uint32_t>(kR) ? static_cast<int32_t>(S.prefix[code] >> sh0)
+                                                               : 0x7FFFFFFF;
+    }
+    __syncthreads();
     // ---- pass 2: decide every token outside its bucket's threshold digit,
     // list the rest
+    // roles are read two iterations ahead of their use (they come from L2)
+    auto roles_of = [&](int i) {
+      const int g = i * NT + tid;
+      return (i < iters && g < ngroups) ? load_roles(v.rp, off, n, g, v.rvec) : 0xFFFFFFFFu;
+    };
+    uint32_t r_next = roles_of(0), r_after = roles_of(1);
     for (int i = 0; i < iters; ++i) {
       const int g = i * NT + tid;
+      const uint32_t rw = r_next;
+      r_next = r_after;
+      r_after = roles_of(i + 2);
       uint32_t m4 = 0, c4 = 0;
       uint32_t ent[4] = {0u, 0u, 0u, 0u};
       if (g < ngroups) {
         const uint4 kv = keys4[g];
         const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
-        const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-          const uint32_t code = static_cast<uint32_t>(S.code_of_role[(rw >> (8 * j)) & 0xFFu]);
-          bool keep = code == kCodeKeep;
-          if (code < static_cast<uint32_t>(kR)) {
-            const uint32_t hb = kk[j] >> sh0, pb = S.prefix[code] >> sh0;
-            keep = hb > pb;
-            if (hb == pb) {
-              c4 |= 1u << j;
-              ent[j] = (code << 16) | static_cast<uint32_t>(4 * g + j);
-            }
+          const uint32_t r = (rw >> (8 * j)) & 0xFFu;
+          const int T = S.first_of_role[r];
+          const int hb = static_cast<int>(kk[j] >> sh0);
+          m4 |= static_cast<uint32_t>(hb > T) << j;
+          if (hb == T) {
+            c4 |= 1u << j;
+            ent[j] = (static_cast<uint32_t>(S.code_of_role[r]) << 16) | static_cast<uint32_t>(4 * g + j);
           }
-          m4 |= static_cast<uint32_t>(keep) << j;
         }
       }
       store_bits(bits, g, nwords, lane, m4);
+      // list slots: lane's rank among the warp's candidates from four ballots
       const int nc = __popc(c4);
-      if (__any_sync(0xffffffffu, nc != 0)) {
-        int incl = nc;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const int t = __shfl_up_sync(0xffffffffu, incl, o);
-          if (lane >= o) incl += t;
-        }
+      const unsigned b1 = __ballot_sync(0xffffffffu, nc >= 1);
+      if (b1 != 0) {
+        const unsigned b2 = __ballot_sync(0xffffffffu, nc >= 2);
+        const unsigned b3 = __ballot_sync(0xffffffffu, nc >= 3);
+        const unsigned b4 = __ballot_sync(0xffffffffu, nc >= 4);
+        const unsigned lt = (1u << lane) - 1u;
         int base = 0;
-        if (lane == 31) base = atomicAdd(&S.list_n, incl);
-        base = __shfl_sync(0xffffffffu, base, 31);
-        int pos = base + incl - nc;
+        if (lane == 0) base = atomicAdd(&S.list_n, __popc(b1) + __popc(b2) + __popc(b3) + __popc(b4));
+        base = __shfl_sync(0xffffffffu, base, 0);
+        int pos = base + __popc(b1 & lt) + __popc(b2 & lt) + __popc(b3 & lt) + __popc(b4 & lt);
 #pragma unroll
         for (int j = 0; j < 4; ++j)
           if ((c4 >> j) & 1u) {

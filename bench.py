@@ -1,9 +1,9 @@
 """Benchmark of the role-conditional KV-eviction hot path on GB300.
 
 One step = the whole path over one batch of synthetic input: SnapKV windowed
-score (pass 1, normalisers, pass 2), the role-conditional selector with the
-max-pool fused into its load, and the K/V gather-compaction, for every
-(layer, sequence, KV head) of the workload.  The default workload is the
+score (both softmax passes in one persistent kernel), the role-conditional
+selector with the max-pool fused into its load, and the K/V gather-compaction,
+for every (layer, sequence, KV head) of the workload.  The default workload is the
 long-context one the headline metric is quoted on: 32 layers, 4 sequences of
 32768 tokens, 32 query / 8 KV heads, head dim 128, W = 64, pool 7, B = 0.10
 (about 17 GB of bf16 K/V resident on the GPU, larger than L2, so no L2 flush
@@ -51,6 +51,12 @@ def max_over_ranks(x: float, world: int) -> float:
     t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def job_throughput(world: int, units_per_rank: float, steps: int, elapsed_ms: float) -> float:
+    """Whole-job rate: every rank processes units_per_rank per step (weak
+    scaling), elapsed_ms is the slowest rank's time for `steps` steps."""
+    return world * units_per_rank * steps / (elapsed_ms / 1e3)
 
 
 def barrier(world: int):
@@ -126,6 +132,14 @@ class ClockSampler:
 
 
 # ------------------------------------------------------- algorithmic counts --
+
+# DRAM bytes (read + write) of one launch of the dominant kernel, from ncu's
+# dram__bytes_read.sum + dram__bytes_write.sum on the same kernel build.  The
+# long workload's fused score launch was captured on its first 2 layers
+# (64 units: 782.5 + 9.8 MB) and scaled by units (x16); any change to that
+# kernel makes this stale, and then it must be measured again.
+MEASURED_TRAFFIC = {("long", "score"): 792.3e6 * 16}
+
 
 def path_counts(w, B):
     """Algorithmic bytes / flops per step of each kernel of the path: K read
@@ -264,7 +278,7 @@ def run_gpu(args):
 
     seq_tokens = w.b * w.n if not w.varlen else sum(w.seqlens)
     ms_step = elapsed_ms / args.steps
-    value = world * seq_tokens * args.steps / (elapsed_ms / 1e3)
+    value = job_throughput(world, seq_tokens, args.steps, elapsed_ms)
 
     peaks = load_peaks()
     counts = path_counts(w, B)
@@ -281,7 +295,8 @@ def run_gpu(args):
                 "unit": "GB/s"}
     roof["frac"] = roof["achieved"] / roof["peak"]
     roof["kernel"] = dom
-    roof["traffic"] = args.traffic
+    roof["traffic"] = (args.traffic if args.traffic is not None
+                       else (MEASURED_TRAFFIC.get((w.name, dom)) if not args.layers else None))
     roof["peak_source"] = peaks["source"] + " (burst)"
     path_frac = counts["path_bytes"] / (ms_step / 1e3) / 1e9 / peaks["hbm_gbs"]
     tensor_util = {nm: counts[nm]["flops"] / (per_kernel[nm] / 1e3) / 1e12 / peaks["bf16_tflops"]
@@ -304,6 +319,10 @@ def run_gpu(args):
         "gpu_launches": len(names) * args.steps,
     }
 
+    if not h2o and not args.no_single_pass:
+        result["single_pass"] = run_single_pass(args, batch, params, w, B, qw, K, V, roles, scores,
+                                                keep, k_out, v_out, ws, status, stream, world,
+                                                seq_tokens)
     if not args.no_e2e:
         result["e2e"] = run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep,
                                 k_out, v_out, status, stream, world, seq_tokens)
@@ -314,6 +333,82 @@ def run_gpu(args):
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def window_lse(w, qw, K):
+    """Natural-log softmax normalisers of the window rows, [L][b][Hq][W] fp32,
+    as an attention prefill would hand them over (computed here once, with
+    fp32 torch matmuls, outside any timed region)."""
+    import torch
+
+    L, b, G, W, d = w.L, w.b, w.G, w.W, w.d
+    lse = torch.zeros((L, b, w.Hq, W), dtype=torch.float32, device=qw.device)
+    lens = list(w.seqlens) if w.varlen else [w.n] * b
+    starts = [0]
+    for x in lens[:-1]:
+        starts.append(starts[-1] + x)
+    scale = 1.0 / math.sqrt(d)
+    for l in range(L):
+        for s in range(b):
+            n = lens[s]
+            if n == 0:
+                continue
+            we = min(W, n)
+            for h in range(w.Hkv):
+                if w.varlen:
+                    k = K[l, starts[s]:starts[s] + n, h].float()
+                else:
+                    k = K[l, s, h, :n].float()
+                q = qw[l, s, h * G:(h + 1) * G, :we].float().reshape(G * we, d)
+                logits = (q @ k.T) * scale
+                pos = (n - we + torch.arange(we, device=q.device)).repeat(G)
+                mask = torch.arange(n, device=q.device)[None, :] > pos[:, None]
+                logits.masked_fill_(mask, float("-inf"))
+                lse[l, s, h * G:(h + 1) * G, :we] = torch.logsumexp(logits, dim=1).reshape(G, we)
+    return lse
+
+
+def run_single_pass(args, batch, params, w, B, qw, K, V, roles, scores, keep, k_out, v_out, ws,
+                    status, stream, world, seq_tokens):
+    """The step with the window normalisers supplied by the caller: the score
+    is one pass over K (no row statistics), then selection and compaction."""
+    import torch
+
+    from paper_2607_13205_gb300 import rolekv as R
+
+    torch.backends.cuda.matmul.allow_tf32 = False
+    lse = window_lse(w, qw, K)
+    torch.cuda.synchronize()
+
+    def step():
+        R.snapkv_score(batch, qw, K, w.W, 1, scores, lse_win=lse, ws=ws, status=status, stream=stream)
+        R.role_alloc_select(batch, scores, roles, params, keep, pool_k=w.pool_k, status=status,
+                            stream=stream)
+        R.kv_compact(batch, K, V, keep, B, k_out, v_out, status=status, stream=stream)
+
+    for _ in range(3):
+        step()
+    steps = max(1, args.steps)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2 * steps + 1)]
+    torch.cuda.synchronize()
+    barrier(world)
+    ev[0].record(stream)
+    for i in range(steps):
+        R.snapkv_score(batch, qw, K, w.W, 1, scores, lse_win=lse, ws=ws, status=status, stream=stream)
+        ev[2 * i + 1].record(stream)
+        R.role_alloc_select(batch, scores, roles, params, keep, pool_k=w.pool_k, status=status,
+                            stream=stream)
+        R.kv_compact(batch, K, V, keep, B, k_out, v_out, status=status, stream=stream)
+        ev[2 * i + 2].record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    total = max_over_ranks(ev[0].elapsed_time(ev[-1]), world)
+    score_ms = sum(ev[2 * i].elapsed_time(ev[2 * i + 1]) for i in range(steps)) / steps
+    if int(status.item()) != 0:
+        raise SystemExit(f"device status {int(status.item())} in the single-pass steps")
+    return {"value": world * seq_tokens * steps / (total / 1e3), "unit": UNIT,
+            "ms_per_step": total / steps, "score_ms": score_ms, "steps": steps,
+            "lse": "window normalisers supplied by the caller (computed once, untimed)"}
 
 
 def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_out, v_out, status,
@@ -505,6 +600,8 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="long")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-single-pass", action="store_true",
+                    help="skip the step with caller-supplied window normalisers")
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)

@@ -24,7 +24,13 @@ matmul / sort as the only library steps:
                            top-ceil(alpha_r B n_kv) per role bucket, alpha
                            renormalised over buckets, slack from saturated
                            buckets redistributed (Section 4.1; Algorithm 1).
-* ``select_unit``       -- per-bucket top-q_r by pooled score (Algorithm 1).
+                           Two more splits: GLOBAL (plain top-k, optional
+                           role ban; Sections 2 and 4) and FAIR (equal
+                           retention rate per role; Section 5
+                           "Fair-eviction baseline").
+* ``select_unit``       -- per-bucket top-q_r by pooled score (Algorithm 1);
+                           ``select_batch`` optionally keeps the last R
+                           tokens first (SnapKV's recency floor, Section 7).
 * ``compact_unit``      -- gather of the kept K/V rows into a dense cache
                            (Section 6 "Systems cost": the compacting
                            implementation the paper describes but does not
@@ -53,6 +59,7 @@ FIXED_ONE = 1_000_000  # fixed-point unit for budgets and alphas (6 decimals)
 
 POLICY_ROLE_QUOTA = 0
 POLICY_GLOBAL = 1
+POLICY_FAIR = 2
 
 
 # ----------------------------------------------------------------------------
@@ -175,7 +182,8 @@ def kept_count(n: int, budget: float) -> int:
 
 
 def role_quotas(counts: Sequence[int], alpha: Sequence[float], budget: float, n: int,
-                policy: int = POLICY_ROLE_QUOTA, ban_mask: int = 0) -> list[int]:
+                policy: int = POLICY_ROLE_QUOTA, ban_mask: int = 0,
+                k_full: int | None = None) -> list[int]:
     """Per-bucket keep counts q_r for one sequence.
 
     ROLE_QUOTA (the combined method, Section 4.1): bucket r gets the share
@@ -190,16 +198,30 @@ def role_quotas(counts: Sequence[int], alpha: Sequence[float], budget: float, n:
     GLOBAL (plain H2O / SnapKV top-k, Section 2; the 'No-X' role ban of
     Section 4 when ban_mask is set): one bucket holding every non-banned
     token; its quota is min(ceil(B n), size) and is reported on bucket 0.
+
+    FAIR (the fair-eviction baseline of Section 5, "Fair-eviction baseline":
+    equal retention rate per role): as ROLE_QUOTA with the weight of every
+    non-banned role equal to its token count, so each role keeps the same
+    fraction of its tokens up to integer rounding; alpha is not used.
+
+    k_full, when given, replaces ceil(B n) as the budget to split (the
+    recency floor of select_batch takes its tokens out of it first).
     """
     R = len(counts)
     counts = [int(c) for c in counts]
-    K_full = kept_count(n, budget) if n > 0 else 0
+    if k_full is not None:
+        K_full = int(k_full)
+    else:
+        K_full = kept_count(n, budget) if n > 0 else 0
     q = [0] * R
     if policy == POLICY_GLOBAL:
         eligible = sum(counts[r] for r in range(R) if not (ban_mask >> r) & 1)
         q[0] = min(K_full, eligible)
         return q
-    a = [0 if (ban_mask >> r) & 1 else to_fixed(alpha[r]) for r in range(R)]
+    if policy == POLICY_FAIR:
+        a = [0 if (ban_mask >> r) & 1 else counts[r] for r in range(R)]
+    else:
+        a = [0 if (ban_mask >> r) & 1 else to_fixed(alpha[r]) for r in range(R)]
     S = [r for r in range(R) if a[r] > 0 and counts[r] > 0]
     K = min(K_full, sum(counts[r] for r in S))
     k_left = K
@@ -225,11 +247,11 @@ def role_quotas(counts: Sequence[int], alpha: Sequence[float], budget: float, n:
 
 
 def bucket_of_tokens(roles: np.ndarray, policy: int, ban_mask: int) -> np.ndarray:
-    """Bucket id of every token: its role (ROLE_QUOTA) or 0 (GLOBAL); -1 for
-    tokens of a banned role."""
+    """Bucket id of every token: its role (ROLE_QUOTA, FAIR) or 0 (GLOBAL);
+    -1 for tokens of a banned role."""
     roles = np.asarray(roles).astype(np.int64)
     banned = ((ban_mask >> roles) & 1).astype(bool)
-    b = roles.copy() if policy == POLICY_ROLE_QUOTA else np.zeros_like(roles)
+    b = np.zeros_like(roles) if policy == POLICY_GLOBAL else roles.copy()
     b[banned] = -1
     return b
 
@@ -356,12 +378,17 @@ def h2o_batch(batch: Batch, q_bits, k_bits, scale: float | None = None,
 
 def select_batch(batch: Batch, unit_scores: dict, roles, n_roles: int, alpha: Sequence[float],
                  key_role: int, alpha_key: float, budget: float,
-                 policy: int = POLICY_ROLE_QUOTA, ban_mask: int = 0):
+                 policy: int = POLICY_ROLE_QUOTA, ban_mask: int = 0, keep_last: int = 0):
     """Role-conditional selection for each unit in ``unit_scores``.
 
     alpha[key_role] is replaced by alpha_key (the method's one tuned knob,
-    Section 4.1).  Returns {unit: (kept_idx padded with -1 to ceil(B n),
-    kept count per role)}.
+    Section 4.1).  keep_last > 0 adds a recency floor (SnapKV's observation
+    window, the part of SnapKV Section 7 finds is not what helps): the last
+    R = min(keep_last, n, ceil(B n)) tokens are kept whatever their score and
+    role, and the remaining ceil(B n) - R slots are split over the earlier
+    tokens exactly as without the floor (roles counted over those tokens
+    only).  Returns {unit: (kept_idx padded with -1 to ceil(B n), kept count
+    per role)}.
     """
     al = [float(np.float32(a)) for a in alpha[:n_roles]]
     if 0 <= key_role < n_roles:
@@ -371,11 +398,15 @@ def select_batch(batch: Batch, unit_scores: dict, roles, n_roles: int, alpha: Se
         _, s, _ = batch.unit(u)
         r = np.asarray(batch.roles(roles, s)).astype(np.int64)
         n = r.shape[0]
-        counts = [int((r == x).sum()) for x in range(n_roles)]
-        q = role_quotas(counts, al, budget, n, policy, ban_mask)
-        bk = bucket_of_tokens(r, policy, ban_mask)
-        idx = select_unit(np.asarray(sc, dtype=np.float64), bk, q)
         width = kept_count(n, budget) if n > 0 else 0
+        forced = min(int(keep_last), n, width)
+        nf = n - forced                              # tokens before the floor
+        counts = [int((r[:nf] == x).sum()) for x in range(n_roles)]
+        q = role_quotas(counts, al, budget, n, policy, ban_mask, k_full=width - forced)
+        bk = bucket_of_tokens(r, policy, ban_mask)
+        bk[nf:] = -1
+        idx = select_unit(np.asarray(sc, dtype=np.float64), bk, q)
+        idx = np.sort(np.concatenate([idx, np.arange(nf, n, dtype=np.int64)]))
         padded = np.full(width, -1, dtype=np.int64)
         padded[:idx.shape[0]] = idx
         per_role = [int((r[idx] == x).sum()) for x in range(n_roles)]

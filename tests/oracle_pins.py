@@ -345,9 +345,84 @@ def pin_varlen_matches_dense(O, rng):
         assert np.allclose(a[u], c[u], rtol=1e-14, atol=0)
 
 
+def pin_fair_quotas(O, rng):
+    """FAIR (equal retention rate per role, Section 5 'Fair-eviction
+    baseline'): the exact rational share of role r is n_r K / N over the
+    non-banned roles; the quotas are its floors, and the K - sum(floors) roles
+    with the largest fractional parts (ties to the lower role) get one more."""
+    for _ in range(300):
+        R = int(rng.integers(1, 9))
+        counts = [int(x) for x in rng.integers(0, 80, size=R)]
+        ban = int(rng.integers(0, 1 << R)) if rng.random() < 0.3 else 0
+        n = sum(counts)
+        if n == 0:
+            continue
+        B = float(rng.choice([0.05, 0.1, 0.2, 0.3, 0.5, 1.0]))
+        q = O.role_quotas(counts, [0.7] * R, B, n, policy=O.POLICY_FAIR, ban_mask=ban)
+        live = [r for r in range(R) if not (ban >> r) & 1 and counts[r] > 0]
+        N = sum(counts[r] for r in live)
+        K = min(math.ceil(Fraction(round(B * 1e6), 10**6) * n), N)
+        assert sum(q) == K
+        if N == 0:
+            assert q == [0] * R
+            continue
+        share = {r: Fraction(counts[r] * K, N) for r in live}
+        floors = {r: math.floor(share[r]) for r in live}
+        extra = K - sum(floors.values())
+        up = sorted(live, key=lambda r: (-(share[r] - floors[r]), r))[:extra]
+        for r in range(R):
+            want = floors[r] + (1 if r in up else 0) if r in share else 0
+            assert q[r] == want, (counts, ban, B, q)
+    # equal rates exactly when the shares are integers: every role keeps B of its tokens
+    q = O.role_quotas([100, 40, 60, 200], [0] * 4, 0.25, 400, policy=O.POLICY_FAIR)
+    assert q == [25, 10, 15, 50]
+
+
+def pin_recency_floor(O, rng):
+    """The recency floor keeps the last R = min(keep_last, n, ceil(B n))
+    tokens and splits the other ceil(B n) - R slots over the earlier tokens:
+    keep_last = 0 is the plain selection, a floor as large as the budget keeps
+    exactly the last ceil(B n) tokens, and on tiny units each bucket's kept
+    subset of the prefix is the brute-force best of its size."""
+    b, n = 2, 240
+    batch = O.Batch(1, b, 2, 1, 8, n)
+    roles = rng.integers(0, 4, size=(b, n)).astype(np.uint8)
+    scores = {u: rng.random(n) for u in range(batch.n_units)}
+    al = [0.25, 0.02, 0.70, 0.05]
+    for B in (0.05, 0.3):
+        plain = O.select_batch(batch, scores, roles, 4, al, 1, 0.02, B)
+        zero = O.select_batch(batch, scores, roles, 4, al, 1, 0.02, B, keep_last=0)
+        K = O.kept_count(n, B)
+        full = O.select_batch(batch, scores, roles, 4, al, 1, 0.02, B, keep_last=10 * n)
+        for u in plain:
+            assert np.array_equal(plain[u][0], zero[u][0])
+            assert np.array_equal(full[u][0], np.arange(n - K, n))
+    for trial in range(30):
+        m = int(rng.integers(8, 15))
+        tb = O.Batch(1, 1, 1, 1, 8, m)
+        rl = rng.integers(0, 3, size=(1, m)).astype(np.uint8)
+        sc = rng.integers(0, 5, size=m).astype(np.float64)
+        B = float(rng.choice([0.3, 0.5, 0.7]))
+        keep = int(rng.integers(1, 4))
+        idx, per = O.select_batch(tb, {0: sc}, rl, 3, [0.5, 0.3, 0.2], -1, 0.0, B, keep_last=keep)[0]
+        K = O.kept_count(m, B)
+        R = min(keep, m, K)
+        kept = [int(t) for t in idx if t >= 0]
+        assert len(kept) == K
+        assert kept[-R:] == list(range(m - R, m))
+        prefix = [t for t in kept if t < m - R]
+        for r in range(3):
+            members = [t for t in range(m - R) if rl[0, t] == r]
+            chosen = tuple(t for t in prefix if rl[0, t] == r)
+            best = min(((-sum(sc[list(sub)]), sub) for sub in itertools.combinations(members, len(chosen))))
+            assert chosen == best[1], (trial, r, chosen, best)
+        assert per == [int((rl[0, kept] == x).sum()) for x in range(3)]
+
+
 ALL_PINS = [
     pin_rows_sum_to_one, pin_snapkv_total, pin_h2o_total, pin_uniform_closed_forms,
     pin_two_level_scale, pin_window_covering_is_h2o, pin_gqa_grouping, pin_maxpool,
     pin_kept_count, pin_quota_golden, pin_quota_waterlevel, pin_key_ban,
     pin_global_is_full_sort, pin_bruteforce_select, pin_compact, pin_varlen_matches_dense,
+    pin_fair_quotas, pin_recency_floor,
 ]

@@ -108,11 +108,12 @@ def _m_round_not_ceil(O):
 
 
 def _m_no_redistribution(O):
-    def role_quotas(counts, alpha, budget, n, policy=0, ban_mask=0):
+    def role_quotas(counts, alpha, budget, n, policy=0, ban_mask=0, k_full=None):
         R = len(counts)
         a = [O.to_fixed(x) for x in alpha]
         E = [r for r in range(R) if a[r] > 0 and counts[r] > 0]
-        K = min(O.kept_count(n, budget), sum(counts[r] for r in E))
+        kf = O.kept_count(n, budget) if k_full is None else k_full
+        K = min(kf, sum(counts[r] for r in E))
         A = sum(a[r] for r in E) or 1
         q = [0] * R
         for r in E:
@@ -124,11 +125,12 @@ def _m_no_redistribution(O):
 def _m_renormalise_all_buckets(O):
     orig = O.role_quotas
 
-    def role_quotas(counts, alpha, budget, n, policy=0, ban_mask=0):
+    def role_quotas(counts, alpha, budget, n, policy=0, ban_mask=0, k_full=None):
         # shares computed over every bucket with alpha > 0, present or not
         R = len(counts)
         a = [O.to_fixed(x) for x in alpha]
-        K = min(O.kept_count(n, budget), sum(c for c, x in zip(counts, a) if x > 0))
+        kf = O.kept_count(n, budget) if k_full is None else k_full
+        K = min(kf, sum(c for c, x in zip(counts, a) if x > 0))
         A = sum(a) or 1
         q = [min(counts[r], (a[r] * K) // A) for r in range(R)]
         return q
@@ -172,6 +174,30 @@ def _m_interleaved_gqa(O):
     O.snapkv_batch = snapkv_batch
 
 
+def _from_source(O, old, new, names):
+    src = open(ORACLE_FILE).read()
+    assert old in src, old
+    ns = {}
+    exec(compile(src.replace(old, new), ORACLE_FILE, "exec"), ns)
+    for nm in names:
+        setattr(O, nm, ns[nm])
+
+
+def _m_fair_uses_alpha(O):
+    _from_source(O, "a = [0 if (ban_mask >> r) & 1 else counts[r] for r in range(R)]",
+                 "a = [0 if (ban_mask >> r) & 1 else to_fixed(alpha[r]) for r in range(R)]",
+                 ["role_quotas"])
+
+
+def _m_floor_outside_budget(O):
+    _from_source(O, "k_full=width - forced)", "k_full=width)", ["select_batch"])
+
+
+def _m_floor_counts_whole_row(O):
+    _from_source(O, "counts = [int((r[:nf] == x).sum())", "counts = [int((r == x).sum())",
+                 ["select_batch"])
+
+
 def _m_compact_off_by_one(O):
     orig = O.compact_unit
     O.compact_unit = lambda rows, idx: orig(rows, np.where(np.asarray(idx) >= 0, np.minimum(np.asarray(idx) + 1, rows.shape[0] - 1), -1))
@@ -181,7 +207,8 @@ MUTATIONS = [
     _m_no_causal, _m_strict_causal, _m_scale_squared, _m_column_normalised, _m_first_window,
     _m_mean_over_heads, _m_h2o_drops_heads, _m_pool_too_wide, _m_pool_one_sided,
     _m_round_not_ceil, _m_no_redistribution, _m_renormalise_all_buckets, _m_remainder_ties_high,
-    _m_ties_to_high_index, _m_interleaved_gqa, _m_compact_off_by_one,
+    _m_ties_to_high_index, _m_interleaved_gqa, _m_compact_off_by_one, _m_fair_uses_alpha,
+    _m_floor_outside_budget, _m_floor_counts_whole_row,
 ]
 
 

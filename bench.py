@@ -203,7 +203,9 @@ def run_gpu(args):
     roles = torch.as_tensor(roles_np, device=dev)
     batch = R.Batch(w.L, w.b, w.Hq, w.Hkv, w.d, w.n, seqlens=list(w.seqlens) if w.varlen else None,
                     device=dev)
-    params = R.select_params(B, I.PAPER_ALPHA, alpha_key=0.0, key_role=I.ROLE_KEY)
+    policy = {"quota": R.POLICY_ROLE_QUOTA, "global": R.POLICY_GLOBAL, "fair": R.POLICY_FAIR}[args.policy]
+    params = R.select_params(B, I.PAPER_ALPHA, alpha_key=0.0, key_role=I.ROLE_KEY, policy=policy,
+                             keep_last=args.keep_last)
     scores = torch.empty(batch.score_shape(), dtype=torch.float32, device=dev)
     keep = torch.empty(batch.kept_shape(B), dtype=torch.int32, device=dev)
     k_out = torch.empty(R.compact_shape(batch, B), dtype=torch.bfloat16, device=dev)
@@ -307,7 +309,9 @@ def run_gpu(args):
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": f"{w.name}: L={w.L} b={w.b} Hq={w.Hq} Hkv={w.Hkv} d={w.d} "
-                               f"N={'varlen<=' if w.varlen else ''}{w.n} W={w.W} pool={w.pool_k} B={B}",
+                               f"N={'varlen<=' if w.varlen else ''}{w.n} W={w.W} pool={w.pool_k} B={B}"
+                               + (f" policy={args.policy}" if args.policy != "quota" else "")
+                               + (f" keep_last={args.keep_last}" if args.keep_last else ""),
                    "global_batch": world * w.b, "seq_len": w.n, "parallelism": f"replicas x{world}",
                    "l2": "inputs larger than L2, no flush"},
         "hbm_path_frac": path_frac,
@@ -327,7 +331,8 @@ def run_gpu(args):
         result["e2e"] = run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep,
                                 k_out, v_out, status, stream, world, seq_tokens)
     if rank == 0 and not args.no_cpu_baseline:
-        result["cpu_baseline"] = cpu_baseline(w, B, args.cpu_seconds, host_inputs=(qw, K, V, roles_np))
+        result["cpu_baseline"] = cpu_baseline(w, B, args.cpu_seconds, host_inputs=(qw, K, V, roles_np),
+                                              policy=args.policy, keep_last=args.keep_last)
     if rank == 0:
         print(json.dumps(result), flush=True)
     if world > 1:
@@ -466,7 +471,10 @@ def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_o
 
 # ------------------------------------------------------ CPU oracle baseline --
 
-def oracle_units(w, B, units, qw_bits, k_bits, v_bits, roles_np):
+POLICY_CODES = {"quota": 0, "global": 1, "fair": 2}
+
+
+def oracle_units(w, B, units, qw_bits, k_bits, v_bits, roles_np, policy="quota", keep_last=0):
     """Score, select and compact the given units with the fp64 oracle."""
     from oracle import rolekv_oracle as O
     from paper_2607_13205_gb300 import inputs as I
@@ -478,7 +486,8 @@ def oracle_units(w, B, units, qw_bits, k_bits, v_bits, roles_np):
     else:
         sc = O.snapkv_batch(ob, qw_bits, k_bits, w.W, w.pool_k, units=units)
         pooled = {u: sc[u][1] for u in sc}
-    sel = O.select_batch(ob, pooled, roles_np, I.N_ROLES, I.PAPER_ALPHA, I.ROLE_KEY, 0.0, B)
+    sel = O.select_batch(ob, pooled, roles_np, I.N_ROLES, I.PAPER_ALPHA, I.ROLE_KEY, 0.0, B,
+                         policy=POLICY_CODES[policy], keep_last=keep_last)
     for u, (idx, _) in sel.items():
         O.compact_unit(ob.kv_rows(k_bits, u), idx)
         O.compact_unit(ob.kv_rows(v_bits, u), idx)
@@ -503,7 +512,7 @@ def _sample_arrays(w, units, host_inputs):
     return qb, kb, vb, roles_np
 
 
-def cpu_baseline(w, B, seconds: float, host_inputs):
+def cpu_baseline(w, B, seconds: float, host_inputs, policy="quota", keep_last=0):
     """The oracle as it stands on this host's cores, on units of layer 0 of
     the same workload until `seconds` of CPU work, extrapolated to a step."""
     U = w.L * w.b * w.Hkv
@@ -517,7 +526,7 @@ def cpu_baseline(w, B, seconds: float, host_inputs):
         if qb is None:
             qb, kb, vb, roles_np = _sample_arrays(w, [u], host_inputs)
         t0 = time.perf_counter()
-        oracle_units(w, B, [u], qb, kb, vb, roles_np)
+        oracle_units(w, B, [u], qb, kb, vb, roles_np, policy, keep_last)
         t_total += time.perf_counter() - t0
         done += 1
         units.append(u)
@@ -568,7 +577,7 @@ def run_reference(args):
         nonlocal nxt
         units = [(nxt + i) % (w1.b * w1.Hkv) for i in range(per_step)]
         nxt += per_step
-        oracle_units(w1, B, units, qb, kb, vb, roles_np)
+        oracle_units(w1, B, units, qb, kb, vb, roles_np, args.policy, args.keep_last)
 
     for _ in range(args.warmup):
         step()
@@ -607,6 +616,10 @@ def main(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-units", type=int, default=2)
     ap.add_argument("--budget", type=float, default=0.0, help="override the workload's budget")
+    ap.add_argument("--policy", choices=["quota", "global", "fair"], default="quota",
+                    help="budget split: role quotas (the method), plain top-k, or fair eviction")
+    ap.add_argument("--keep-last", type=int, default=0,
+                    help="recency floor: always keep each sequence's last tokens")
     ap.add_argument("--layers", type=int, default=0,
                     help="override the layer count (smaller cases for profiling)")
     ap.add_argument("--traffic", type=float, default=None,

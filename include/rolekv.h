@@ -74,6 +74,7 @@ extern "C" {
 
 #define ROLEKV_POLICY_ROLE_QUOTA 0  /* the combined method (Section 4.1)       */
 #define ROLEKV_POLICY_GLOBAL 1      /* plain top-k, optional role ban (Sec. 4) */
+#define ROLEKV_POLICY_FAIR 2        /* equal retention rate per role (Sec. 5)  */
 
 #define ROLEKV_MAX_ROLES 8
 #define ROLEKV_SELECT_MAX_N 40960   /* largest sequence role_alloc_select takes */
@@ -107,7 +108,15 @@ typedef struct rolekv_batch {
  *              ROLEKV_POLICY_GLOBAL: one bucket of all non-banned tokens, top
  *              min(ceil(B*n), eligible) by score (plain H2O / SnapKV top-k;
  *              with ban_mask it is the counterfactual 'No-X' ban of Section 4).
+ *              ROLEKV_POLICY_FAIR: the fair-eviction baseline of Section 5
+ *              (equal retention rate per role): as ROLE_QUOTA with every
+ *              non-banned role weighted by its token count; alpha is unused.
  *   ban_mask   bit r set: role r keeps nothing.
+ *   keep_last  recency floor (SnapKV's observation window, Section 7): the
+ *              last R = min(keep_last, n, ceil(B*n)) tokens of each sequence
+ *              are kept whatever their score and role; the other
+ *              ceil(B*n) - R slots are split as above over the earlier tokens,
+ *              whose roles alone are counted.  0: no floor.
  * Within a bucket the highest scores win and equal scores go to the lower
  * token index. */
 typedef struct rolekv_select_params {
@@ -118,6 +127,7 @@ typedef struct rolekv_select_params {
   float budget;
   int32_t policy;
   uint32_t ban_mask;
+  int32_t keep_last;             /* >= 0                                      */
 } rolekv_select_params;
 
 /* Number of kept slots of an n-token sequence at budget B: ceil(B*n) with B in

@@ -74,6 +74,7 @@ struct SelectArgs {
   int64_t budget_fx;
   int32_t policy;
   uint32_t ban_mask;
+  int32_t keep_last;                    // recency floor (tokens), 0 = none
   int32_t* keep_idx;
   uint8_t* keep_mask;
   int32_t* kept_per_role;

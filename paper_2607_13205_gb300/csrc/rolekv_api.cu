@@ -382,8 +382,10 @@ int fill_select(const BatchInfo& bi, const rolekv_batch* bt, const rolekv_select
     return fail(ROLEKV_ERR_UNSUPPORTED, "n_roles=%d outside 1..%d", sp->n_roles, ROLEKV_MAX_ROLES);
   if (!(sp->budget > 0.f) || sp->budget > 1.f)
     return fail(ROLEKV_ERR_INVALID_ARG, "budget %g outside (0, 1]", static_cast<double>(sp->budget));
-  if (sp->policy != ROLEKV_POLICY_ROLE_QUOTA && sp->policy != ROLEKV_POLICY_GLOBAL)
+  if (sp->policy != ROLEKV_POLICY_ROLE_QUOTA && sp->policy != ROLEKV_POLICY_GLOBAL &&
+      sp->policy != ROLEKV_POLICY_FAIR)
     return fail(ROLEKV_ERR_INVALID_ARG, "unknown policy %d", sp->policy);
+  if (sp->keep_last < 0) return fail(ROLEKV_ERR_INVALID_ARG, "keep_last=%d must be >= 0", sp->keep_last);
   if (sp->key_role >= sp->n_roles) return fail(ROLEKV_ERR_INVALID_ARG, "key_role %d >= n_roles", sp->key_role);
   if (bi.n_max > ROLEKV_SELECT_MAX_N)
     return fail(ROLEKV_ERR_UNSUPPORTED, "n_max=%d exceeds the %d tokens the selector holds", bi.n_max,
@@ -400,6 +402,7 @@ int fill_select(const BatchInfo& bi, const rolekv_batch* bt, const rolekv_select
   a->budget_fx = to_fixed(sp->budget);
   a->policy = sp->policy;
   a->ban_mask = sp->ban_mask;
+  a->keep_last = sp->keep_last;
   for (int r = 0; r < ROLEKV_MAX_ROLES; ++r) {
     float al = r < sp->n_roles ? sp->alpha[r] : 0.f;
     if (r == sp->key_role) al = sp->alpha_key;

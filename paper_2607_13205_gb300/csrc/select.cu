@@ -103,6 +103,7 @@ struct SelShared {
   int32_t hist[kR][256];
   int32_t warp_tot[32];
   int32_t kept_role[kR];
+  int32_t floor_role[kR];  // recency-floor tokens per role
   uint32_t ties[kTieCap];  // (bucket << 16) | slot of keys equal to a threshold
   uint32_t top_and, top_or;
   int32_t list_n, tie_n;
@@ -144,14 +145,26 @@ struct UnitView {
   const float* sp;
   const uint8_t* rp;
   int off, n, ngroups;
+  int nf;          // tokens before the recency floor (the floor is [nf, n))
   bool rvec;
 };
+
+// Bits j of the slots 4g+j (first token s0 = 4g - off) inside the recency
+// floor [nf, n).
+__device__ __forceinline__ uint32_t floor_bits(int s0, int nf, int n) {
+  if (s0 + 4 <= nf || s0 >= n) return 0u;
+  uint32_t m = 0;
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+    if (s0 + j >= nf && s0 + j < n) m |= 1u << j;
+  return m;
+}
 
 // Pass 1 for a pool half-width HW known at compile time.
 template <int HW, int NT>
 __device__ __forceinline__ void pass1(const UnitView& v, int n_roles, int nb, uint4* keys4,
-                                      uint32_t* hist16, bool& nan_hint, uint32_t& top_and,
-                                      uint32_t& top_or) {
+                                      uint32_t* hist16, int32_t* floor_role, bool& nan_hint,
+                                      uint32_t& top_and, uint32_t& top_or) {
   constexpr int NB = (HW + 3) / 4;   // neighbour groups on each side
   const int sh0 = 31 - nb;
   const uint32_t bmask = (1u << nb) - 1u;
@@ -184,10 +197,13 @@ __device__ __forceinline__ void pass1(const UnitView& v, int n_roles, int nb, ui
     }
     keys4[g] = make_uint4(k[0], k[1], k[2], k[3]);
     const uint32_t rw = load_roles(v.rp, v.off, v.n, g, v.rvec);
+    const uint32_t fb = floor_bits(4 * g - v.off, v.nf, v.n);
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       const uint32_t r = (rw >> (8 * j)) & 0xFFu;
-      if (r < static_cast<uint32_t>(n_roles)) {
+      if ((fb >> j) & 1u) {                      // recency floor: kept, counted apart
+        if (r < static_cast<uint32_t>(n_roles)) atomicAdd(&floor_role[r], 1);
+      } else if (r < static_cast<uint32_t>(n_roles)) {
         top_and &= k[j];
         top_or |= k[j];
         const uint32_t bin = (k[j] >> sh0) & bmask;
@@ -214,7 +230,9 @@ __device__ void quotas_warp(const SelectArgs& a, int lane, int64_t K_full, SelSh
   const bool valid = r < a.n_roles;
   const bool banned = valid && ((a.ban_mask >> r) & 1u);
   const int64_t cnt = valid ? S.count[r] : 0;
-  const int64_t alpha = r < kR ? a.alpha_fx[r] : 0;
+  // FAIR: every non-banned role weighted by its own token count
+  const int64_t alpha = (a.policy == ROLEKV_POLICY_FAIR) ? ((valid && !banned) ? cnt : 0)
+                                                         : a.alpha_fx[r];
   int64_t q = 0, bsize = 0;
   if (a.policy == ROLEKV_POLICY_GLOBAL) {
     const int64_t elig = sum8((valid && !banned) ? cnt : 0);
@@ -495,6 +513,9 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
   const int nslots = v.off + n;
   v.ngroups = (nslots + 3) >> 2;
   v.rvec = ((reinterpret_cast<uintptr_t>(v.rp) - static_cast<uintptr_t>(v.off)) & 3u) == 0;
+  const int64_t n_floor = a.keep_last < n ? (a.keep_last < K_s ? a.keep_last : K_s)
+                                          : (n < K_s ? n : K_s);
+  v.nf = n - static_cast<int>(n_floor);
   const int off = v.off, ngroups = v.ngroups;
   const int nwords = (nslots + 31) >> 5;
   const int iters = (ngroups + NT - 1) / NT;
@@ -511,6 +532,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
   if (tid < kR) {
     S.count[tid] = 0;
     S.kept_role[tid] = 0;
+    S.floor_role[tid] = 0;
   }
   if (tid == 0) {
     S.nan_hint = 0;
@@ -551,14 +573,14 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
     bool nan_hint = false;
     uint32_t tand = 0xFFFFFFFFu, tor = 0u;
     switch (a.pool_k >> 1) {
-      case 0: pass1<0, NT>(v, a.n_roles, nb, keys4, hist16, nan_hint, tand, tor); break;
-      case 1: pass1<1, NT>(v, a.n_roles, nb, keys4, hist16, nan_hint, tand, tor); break;
-      case 2: pass1<2, NT>(v, a.n_roles, nb, keys4, hist16, nan_hint, tand, tor); break;
-      case 3: pass1<3, NT>(v, a.n_roles, nb, keys4, hist16, nan_hint, tand, tor); break;
-      case 4: pass1<4, NT>(v, a.n_roles, nb, keys4, hist16, nan_hint, tand, tor); break;
-      case 5: pass1<5, NT>(v, a.n_roles, nb, keys4, hist16, nan_hint, tand, tor); break;
-      case 6: pass1<6, NT>(v, a.n_roles, nb, keys4, hist16, nan_hint, tand, tor); break;
-      default: pass1<7, NT>(v, a.n_roles, nb, keys4, hist16, nan_hint, tand, tor); break;
+      case 0: pass1<0, NT>(v, a.n_roles, nb, keys4, hist16, S.floor_role, nan_hint, tand, tor); break;
+      case 1: pass1<1, NT>(v, a.n_roles, nb, keys4, hist16, S.floor_role, nan_hint, tand, tor); break;
+      case 2: pass1<2, NT>(v, a.n_roles, nb, keys4, hist16, S.floor_role, nan_hint, tand, tor); break;
+      case 3: pass1<3, NT>(v, a.n_roles, nb, keys4, hist16, S.floor_role, nan_hint, tand, tor); break;
+      case 4: pass1<4, NT>(v, a.n_roles, nb, keys4, hist16, S.floor_role, nan_hint, tand, tor); break;
+      case 5: pass1<5, NT>(v, a.n_roles, nb, keys4, hist16, S.floor_role, nan_hint, tand, tor); break;
+      case 6: pass1<6, NT>(v, a.n_roles, nb, keys4, hist16, S.floor_role, nan_hint, tand, tor); break;
+      default: pass1<7, NT>(v, a.n_roles, nb, keys4, hist16, S.floor_role, nan_hint, tand, tor); break;
     }
     tand = __reduce_and_sync(0xffffffffu, tand);
     tor = __reduce_or_sync(0xffffffffu, tor);
@@ -605,7 +627,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
   __syncthreads();
 
   // ---- quotas and the role -> code table
-  if (warp == 0) quotas_warp(a, lane, K_s, S);
+  if (warp == 0) quotas_warp(a, lane, K_s - n_floor, S);
   __syncthreads();
   for (int x = tid; x < 256; x += NT) {
     uint32_t code = kCodeDrop;
@@ -663,17 +685,19 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
       if (g < ngroups) {
         const uint4 kv = keys4[g];
         const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
+        const uint32_t fb = floor_bits(4 * g - off, v.nf, n);
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           const uint32_t r = (rw >> (8 * j)) & 0xFFu;
           const int T = S.first_of_role[r];
           const int hb = static_cast<int>(kk[j] >> sh0);
           m4 |= static_cast<uint32_t>(hb > T) << j;
-          if (hb == T) {
+          if (hb == T && !((fb >> j) & 1u)) {
             c4 |= 1u << j;
             ent[j] = (static_cast<uint32_t>(S.code_of_role[r]) << 16) | static_cast<uint32_t>(4 * g + j);
           }
         }
+        m4 |= fb;                                  // the recency floor is kept
       }
       store_bits(bits, g, nwords, lane, m4);
       // list slots: lane's rank among the warp's candidates from four ballots
@@ -771,10 +795,11 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
         const uint4 kv = keys4[g];
         const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
         const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
+        const uint32_t fb = floor_bits(4 * g - off, v.nf, n);
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           const uint32_t c = static_cast<uint32_t>(S.code_of_role[(rw >> (8 * j)) & 0xFFu]);
-          if (c >= static_cast<uint32_t>(kR)) continue;
+          if (c >= static_cast<uint32_t>(kR) || ((fb >> j) & 1u)) continue;
           if (round > 0 && (kk[j] >> (shift + 8)) != (S.prefix[c] >> (shift + 8))) continue;
           atomicAdd(&S.hist[c][(kk[j] >> shift) & 0xFFu], 1);
         }
@@ -796,6 +821,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
           const bool keep = (c < static_cast<uint32_t>(kR)) ? (kk[j] >= S.thr[c]) : (c == kCodeKeep);
           m4 |= static_cast<uint32_t>(keep) << j;
         }
+        m4 |= floor_bits(4 * g - off, v.nf, n);    // the recency floor is kept
       }
       store_bits(bits, g, nwords, lane, m4);
     }
@@ -818,9 +844,11 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
           const uint4 kv = keys4[g];
           const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
           const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
+          const uint32_t fb = floor_bits(4 * g - off, v.nf, n);
 #pragma unroll
           for (int j = 0; j < 4; ++j)
-            if (S.code_of_role[(rw >> (8 * j)) & 0xFFu] == b && kk[j] == P) mk |= 1u << (4 * gg + j);
+            if (S.code_of_role[(rw >> (8 * j)) & 0xFFu] == b && kk[j] == P && !((fb >> j) & 1u))
+              mk |= 1u << (4 * gg + j);
         }
         return mk;
       };
@@ -879,7 +907,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
     }
     if (tid < a.n_roles)
       a.kept_per_role[static_cast<int64_t>(u) * a.n_roles + tid] =
-          count_roles ? S.kept_role[tid] : S.quota[tid];
+          count_roles ? S.kept_role[tid] : S.quota[tid] + S.floor_role[tid];
   }
   if (tid == 0 && S.nan_seen && a.status != nullptr) atomicOr(a.status, ROLEKV_STATUS_NONFINITE);
 }

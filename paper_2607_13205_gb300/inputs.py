@@ -39,6 +39,14 @@ N_ROLES = 4
 PAPER_ALPHA = (0.25, 0.0, 0.70, 0.05)
 ALPHA_KEY_SAFE = 0.02   # the cross-model safe default (Section 5)
 
+# The paper's six-label taxonomy (Section 3) with its policy (Section 4.1);
+# HEADER, a schema label like KEY, takes alpha_KEY as well.
+SIX_ROLE_NAMES = ("KEY", "VALUE", "DELIM", "HEADER", "PROSE", "WS")
+
+
+def paper_alpha6(alpha_key: float) -> tuple:
+    return (alpha_key, 0.70, 0.20, alpha_key, 0.05, 0.05)
+
 SINK_SHIFT = 8.0    # a
 KEY_SHIFT = 0.75    # b
 QUERY_SHIFT = 4.0   # c

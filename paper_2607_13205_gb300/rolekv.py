@@ -18,7 +18,7 @@ _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "librolekv.
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA = 0, 1, 2, 3, 4
 STATUS_NONFINITE, STATUS_BAD_INDEX, STATUS_TIMEOUT = 1, 2, 4
-POLICY_ROLE_QUOTA, POLICY_GLOBAL = 0, 1
+POLICY_ROLE_QUOTA, POLICY_GLOBAL, POLICY_FAIR = 0, 1, 2
 MAX_ROLES = 8
 SELECT_MAX_N = 40960
 OP_SNAPKV, OP_H2O, OP_COMPRESS = 0, 1, 2
@@ -46,7 +46,7 @@ class SelectParams(ctypes.Structure):
     _fields_ = [("n_roles", ctypes.c_int32), ("alpha", ctypes.c_float * MAX_ROLES),
                 ("key_role", ctypes.c_int32), ("alpha_key", ctypes.c_float),
                 ("budget", ctypes.c_float), ("policy", ctypes.c_int32),
-                ("ban_mask", ctypes.c_uint32)]
+                ("ban_mask", ctypes.c_uint32), ("keep_last", ctypes.c_int32)]
 
 
 _lib = None
@@ -183,9 +183,10 @@ def tensor_desc(t: torch.Tensor, packed: bool = False) -> Tensor:
 
 
 def select_params(budget: float, alpha: Sequence[float], alpha_key: float = 0.0, key_role: int = 1,
-                  policy: int = POLICY_ROLE_QUOTA, ban_mask: int = 0) -> SelectParams:
+                  policy: int = POLICY_ROLE_QUOTA, ban_mask: int = 0,
+                  keep_last: int = 0) -> SelectParams:
     al = (ctypes.c_float * MAX_ROLES)(*([float(x) for x in alpha] + [0.0] * (MAX_ROLES - len(alpha))))
-    return SelectParams(len(alpha), al, key_role, alpha_key, budget, policy, ban_mask)
+    return SelectParams(len(alpha), al, key_role, alpha_key, budget, policy, ban_mask, keep_last)
 
 
 # ----------------------------------------------------------------- entry points

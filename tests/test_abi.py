@@ -99,6 +99,13 @@ def test_host_rejects_bad_arguments(lib):
     p_neg = R.select_params(0.1, [0.25, 0.0, -0.7, 0.05])
     rc = lib.role_alloc_select(ctypes.byref(b), f, f, ctypes.byref(p_neg), 1, f, None, None, None, None)
     assert rc == R.ERR_INVALID_ARG
+    p_pol = R.select_params(0.1, [0.25, 0.0, 0.7, 0.05], policy=3)
+    rc = lib.role_alloc_select(ctypes.byref(b), f, f, ctypes.byref(p_pol), 1, f, None, None, None, None)
+    assert rc == R.ERR_INVALID_ARG                                      # unknown policy
+    p_floor = R.select_params(0.1, [0.25, 0.0, 0.7, 0.05], keep_last=-1)
+    rc = lib.role_alloc_select(ctypes.byref(b), f, f, ctypes.byref(p_floor), 1, f, None, None, None, None)
+    assert rc == R.ERR_INVALID_ARG                                      # negative floor
+    assert b"keep_last" in lib.rolekv_last_error()
     big = _batch(n_max=R.SELECT_MAX_N + 1)
     rc = lib.role_alloc_select(ctypes.byref(big), f, f, ctypes.byref(p), 1, f, None, None, None, None)
     assert rc == R.ERR_UNSUPPORTED

@@ -128,30 +128,41 @@ def _tied_scores(shape, seed):
     return (torch.randint(0, 64, shape, generator=g).float() / 8.0).to(DEV)
 
 
+VARLEN4 = _w("ragged", L=2, b=4, Hq=8, Hkv=2, n=3000, seqlens=(3000, 0, 5, 1200))
+
 SELECT_CASES = [
-    # (name, workload, budget, alpha_key, policy, ban_mask, pool_k)
+    # (name, workload, budget, alpha_key, policy, ban_mask, pool_k[, keep_last])
     ("combined_b05", _w("llama8b", L=2, b=2, Hq=8, Hkv=2, n=5000), 0.05, 0.0, 0, 0, 1),
     ("combined_b10_pool7", _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=5000), 0.10, 0.02, 0, 0, 7),
     ("combined_b50", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=3001), 0.50, 0.0, 0, 0, 1),
     ("full_budget", _w("llama8b", L=1, b=1, Hq=4, Hkv=1, n=777), 1.0, 0.0, 0, 0, 3),
     ("global_no_key", _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=4000), 0.30, 0.0, 1, 1 << I.ROLE_KEY, 1),
     ("global_plain", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=4000), 0.20, 0.0, 1, 0, 5),
-    ("varlen", _w("ragged", L=2, b=4, Hq=8, Hkv=2, n=3000, seqlens=(3000, 0, 5, 1200)), 0.10, 0.0, 0, 0, 7),
+    ("varlen", VARLEN4, 0.10, 0.0, 0, 0, 7),
     ("mid_n", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=12001), 0.10, 0.02, 0, 0, 7),
     ("mid_n_global_pool15", _w("llama8b", L=1, b=1, Hq=4, Hkv=1, n=9999), 0.10, 0.0, 1, 0, 15),
     ("max_n", _w("long", L=1, b=1, Hq=4, Hkv=1, n=R.SELECT_MAX_N), 0.10, 0.0, 0, 0, 7),
+    # fair eviction (equal retention rate per role) and the recency floor
+    ("fair_pool7", _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=5000), 0.10, 0.0, R.POLICY_FAIR, 0, 7),
+    ("fair_no_key_varlen", VARLEN4, 0.20, 0.0, R.POLICY_FAIR, 1 << I.ROLE_KEY, 7),
+    ("floor64_combined", _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=5000), 0.10, 0.02, 0, 0, 7, 64),
+    ("floor32_global_varlen", VARLEN4, 0.10, 0.0, R.POLICY_GLOBAL, 0, 3, 32),
+    ("floor_over_budget", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=3001), 0.05, 0.0, 0, 0, 7, 1000),
+    ("floor_fair_mid_n", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=12001), 0.10, 0.0, R.POLICY_FAIR, 0, 7, 64),
+    ("floor_max_n", _w("long", L=1, b=1, Hq=4, Hkv=1, n=R.SELECT_MAX_N), 0.10, 0.0, 0, 0, 7, 64),
 ]
 
 
 @pytest.mark.parametrize("case", SELECT_CASES, ids=[c[0] for c in SELECT_CASES])
 def test_role_alloc_select_bit_exact(case):
-    name, w, B, akey, policy, ban, pool_k = case
+    name, w, B, akey, policy, ban, pool_k = case[:7]
+    keep_last = case[7] if len(case) > 7 else 0
     roles_np = I.workload_roles(w, 2)
     batch = lib_batch(w, DEV)
     scores = _tied_scores(batch.score_shape(), 5)
     roles = torch.as_tensor(roles_np, device=DEV)
     params = R.select_params(B, I.PAPER_ALPHA, alpha_key=akey, key_role=I.ROLE_KEY, policy=policy,
-                             ban_mask=ban)
+                             ban_mask=ban, keep_last=keep_last)
     keep = torch.full(batch.kept_shape(B), -7, dtype=torch.int32, device=DEV)
     mask = torch.full(batch.score_shape(), 9, dtype=torch.uint8, device=DEV)
     per_role = torch.full((batch.n_units, I.N_ROLES), -1, dtype=torch.int32, device=DEV)
@@ -167,7 +178,7 @@ def test_role_alloc_select_bit_exact(case):
         s = ob.score_view(sc, u).astype(np.float64)
         unit_scores[u] = O.maxpool1d(s, pool_k) if s.size else s
     ref = O.select_batch(ob, unit_scores, roles_np, I.N_ROLES, I.PAPER_ALPHA, I.ROLE_KEY, akey, B,
-                         policy, ban)
+                         policy, ban, keep_last=keep_last)
     cu_kept = ob.kept_offsets(B)
     keep_np, mask_np, pr = keep.cpu().numpy(), mask.cpu().numpy(), per_role.cpu().numpy()
     for u, (idx, per) in ref.items():
@@ -182,8 +193,37 @@ def test_role_alloc_select_bit_exact(case):
         expect = np.zeros(m.shape, dtype=np.uint8)
         expect[idx[idx >= 0]] = 1
         assert np.array_equal(m, expect), f"{name} unit {u} mask"
-        if akey == 0.0 and policy == 0:
+        if akey == 0.0 and policy == 0 and keep_last == 0:
             assert per[I.ROLE_KEY] == 0
+
+
+@pytest.mark.parametrize("akey", [0.0, 0.02])
+def test_select_six_role_taxonomy(akey):
+    """The paper's six labels (KEY, VALUE, DELIM, HEADER, PROSE, WS) with its
+    policy; a few tokens carry labels outside the six (no bucket)."""
+    w = _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=6001)
+    g = np.random.default_rng(8)
+    roles_np = g.choice(8, size=(w.b, w.n), p=[0.25, 0.2, 0.3, 0.05, 0.1, 0.08, 0.01, 0.01]).astype(np.uint8)
+    batch = lib_batch(w, DEV)
+    scores = _tied_scores(batch.score_shape(), 13)
+    alpha = I.paper_alpha6(akey)
+    B = 0.10
+    params = R.select_params(B, alpha, alpha_key=akey, key_role=0)
+    keep = torch.empty(batch.kept_shape(B), dtype=torch.int32, device=DEV)
+    per_role = torch.empty((batch.n_units, 6), dtype=torch.int32, device=DEV)
+    R.role_alloc_select(batch, scores, torch.as_tensor(roles_np, device=DEV), params, keep, pool_k=7,
+                        kept_per_role=per_role)
+    torch.cuda.synchronize()
+    ob = oracle_batch(w)
+    sc = scores.cpu().numpy()
+    unit_scores = {u: O.maxpool1d(ob.score_view(sc, u).astype(np.float64), 7) for u in range(ob.n_units)}
+    ref = O.select_batch(ob, unit_scores, roles_np, 6, alpha, 0, akey, B)
+    got, pr = keep.cpu().numpy().reshape(ob.n_units, -1), per_role.cpu().numpy()
+    for u, (idx, per) in ref.items():
+        assert np.array_equal(got[u], idx), f"unit {u}"
+        assert list(pr[u]) == per
+        if akey == 0.0:
+            assert per[0] == 0 and per[3] == 0
 
 
 @pytest.mark.parametrize("pool_k", [1, 7])

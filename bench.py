@@ -138,10 +138,11 @@ class ClockSampler:
 # long workload's fused score launch was captured on its first 2 layers
 # (64 units: 782.5 + 9.8 MB) and scaled by units (x16); any change to that
 # kernel makes this stale, and then it must be measured again.
-MEASURED_TRAFFIC = {("long", "score"): 792.3e6 * 16}
+MEASURED_TRAFFIC = {("long", "snapkv", "score"): 792.3e6 * 16,
+                    ("long", "quest", "score"): (541.1e6 + 5.8e6) * 16}
 
 
-def path_counts(w, B):
+def path_counts(w, B, score_kind="snapkv"):
     """Algorithmic bytes / flops per step of each kernel of the path: K read
     once, the queries, the pre-pool score written and read once, the kept K/V
     rows read and written, the kept index written and read.  Variable-length
@@ -167,6 +168,9 @@ def path_counts(w, B):
     kbytes = U * n * d * 2
     qbytes = U * rows * d * 2
     flops = 2.0 * U * rows * n * d
+    if score_kind == "quest":
+        # one pass over K for the page bounds, no contraction
+        flops = 0.0
     return {
         # both passes in one kernel: K crosses HBM once, the QK^T is done twice
         "score": {"bytes": kbytes + qbytes + U * n * 4, "flops": 2 * flops},
@@ -220,6 +224,8 @@ def run_gpu(args):
     def score():
         if h2o:
             R.h2o_score(batch, qw, K, scores, ws=ws, status=status, stream=stream)
+        elif args.score == "quest":
+            R.quest_score(batch, qw, K, w.W, args.page, scores, stream=stream)
         else:
             # pool_k = 1: the pre-pool scores go straight out; the selector pools
             R.snapkv_score(batch, qw, K, w.W, 1, scores, ws=ws, status=status, stream=stream)
@@ -283,7 +289,7 @@ def run_gpu(args):
     value = job_throughput(world, seq_tokens, args.steps, elapsed_ms)
 
     peaks = load_peaks()
-    counts = path_counts(w, B)
+    counts = path_counts(w, B, args.score)
     dom = max(names, key=lambda k: per_kernel[k])
     dk = counts[dom]
     t_dom = per_kernel[dom] / 1e3
@@ -298,7 +304,7 @@ def run_gpu(args):
     roof["frac"] = roof["achieved"] / roof["peak"]
     roof["kernel"] = dom
     roof["traffic"] = (args.traffic if args.traffic is not None
-                       else (MEASURED_TRAFFIC.get((w.name, dom)) if not args.layers else None))
+                       else (MEASURED_TRAFFIC.get((w.name, args.score, dom)) if not args.layers else None))
     roof["peak_source"] = peaks["source"] + " (burst)"
     path_frac = counts["path_bytes"] / (ms_step / 1e3) / 1e9 / peaks["hbm_gbs"]
     tensor_util = {nm: counts[nm]["flops"] / (per_kernel[nm] / 1e3) / 1e12 / peaks["bf16_tflops"]
@@ -310,12 +316,13 @@ def run_gpu(args):
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": f"{w.name}: L={w.L} b={w.b} Hq={w.Hq} Hkv={w.Hkv} d={w.d} "
                                f"N={'varlen<=' if w.varlen else ''}{w.n} W={w.W} pool={w.pool_k} B={B}"
+                               + (f" score=quest page={args.page}" if args.score == "quest" else "")
                                + (f" policy={args.policy}" if args.policy != "quota" else "")
                                + (f" keep_last={args.keep_last}" if args.keep_last else ""),
                    "global_batch": world * w.b, "seq_len": w.n, "parallelism": f"replicas x{world}",
                    "l2": "inputs larger than L2, no flush"},
         "hbm_path_frac": path_frac,
-        "tensor_frac_of_measured_peak": tensor_util,
+        "tensor_frac_of_measured_peak": tensor_util or None,
         "per_kernel_ms": per_kernel,
         "unit_tokens_per_s": world * w.L * w.Hkv * seq_tokens * args.steps / (elapsed_ms / 1e3),
         "roofline": roof,
@@ -323,7 +330,7 @@ def run_gpu(args):
         "gpu_launches": len(names) * args.steps,
     }
 
-    if not h2o and not args.no_single_pass:
+    if not h2o and args.score == "snapkv" and not args.no_single_pass:
         result["single_pass"] = run_single_pass(args, batch, params, w, B, qw, K, V, roles, scores,
                                                 keep, k_out, v_out, ws, status, stream, world,
                                                 seq_tokens)
@@ -332,7 +339,8 @@ def run_gpu(args):
                                 k_out, v_out, status, stream, world, seq_tokens)
     if rank == 0 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(w, B, args.cpu_seconds, host_inputs=(qw, K, V, roles_np),
-                                              policy=args.policy, keep_last=args.keep_last)
+                                              policy=args.policy, keep_last=args.keep_last,
+                                              score_kind=args.score, page=args.page)
     if rank == 0:
         print(json.dumps(result), flush=True)
     if world > 1:
@@ -474,7 +482,8 @@ def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_o
 POLICY_CODES = {"quota": 0, "global": 1, "fair": 2}
 
 
-def oracle_units(w, B, units, qw_bits, k_bits, v_bits, roles_np, policy="quota", keep_last=0):
+def oracle_units(w, B, units, qw_bits, k_bits, v_bits, roles_np, policy="quota", keep_last=0,
+                 score_kind="snapkv", page=16):
     """Score, select and compact the given units with the fp64 oracle."""
     from oracle import rolekv_oracle as O
     from paper_2607_13205_gb300 import inputs as I
@@ -483,6 +492,8 @@ def oracle_units(w, B, units, qw_bits, k_bits, v_bits, roles_np, policy="quota",
     if w.kind == "h2o":
         sc = O.h2o_batch(ob, qw_bits, k_bits, units=units)
         pooled = sc
+    elif score_kind == "quest":
+        pooled = O.quest_batch(ob, qw_bits, k_bits, w.W, page, units=units)
     else:
         sc = O.snapkv_batch(ob, qw_bits, k_bits, w.W, w.pool_k, units=units)
         pooled = {u: sc[u][1] for u in sc}
@@ -512,7 +523,8 @@ def _sample_arrays(w, units, host_inputs):
     return qb, kb, vb, roles_np
 
 
-def cpu_baseline(w, B, seconds: float, host_inputs, policy="quota", keep_last=0):
+def cpu_baseline(w, B, seconds: float, host_inputs, policy="quota", keep_last=0, score_kind="snapkv",
+                 page=16):
     """The oracle as it stands on this host's cores, on units of layer 0 of
     the same workload until `seconds` of CPU work, extrapolated to a step."""
     U = w.L * w.b * w.Hkv
@@ -526,7 +538,7 @@ def cpu_baseline(w, B, seconds: float, host_inputs, policy="quota", keep_last=0)
         if qb is None:
             qb, kb, vb, roles_np = _sample_arrays(w, [u], host_inputs)
         t0 = time.perf_counter()
-        oracle_units(w, B, [u], qb, kb, vb, roles_np, policy, keep_last)
+        oracle_units(w, B, [u], qb, kb, vb, roles_np, policy, keep_last, score_kind, page)
         t_total += time.perf_counter() - t0
         done += 1
         units.append(u)
@@ -577,7 +589,8 @@ def run_reference(args):
         nonlocal nxt
         units = [(nxt + i) % (w1.b * w1.Hkv) for i in range(per_step)]
         nxt += per_step
-        oracle_units(w1, B, units, qb, kb, vb, roles_np, args.policy, args.keep_last)
+        oracle_units(w1, B, units, qb, kb, vb, roles_np, args.policy, args.keep_last, args.score,
+                     args.page)
 
     for _ in range(args.warmup):
         step()
@@ -616,6 +629,9 @@ def main(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-units", type=int, default=2)
     ap.add_argument("--budget", type=float, default=0.0, help="override the workload's budget")
+    ap.add_argument("--score", choices=["snapkv", "quest"], default="snapkv",
+                    help="score of the SnapKV workloads: windowed mass, or the Quest page bound")
+    ap.add_argument("--page", type=int, default=16, help="tokens per page of the Quest bound")
     ap.add_argument("--policy", choices=["quota", "global", "fair"], default="quota",
                     help="budget split: role quotas (the method), plain top-k, or fair eviction")
     ap.add_argument("--keep-last", type=int, default=0,

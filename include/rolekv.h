@@ -191,6 +191,20 @@ int snapkv_score_noalloc(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_
                          float* scores, float* scores_prepool, int32_t* status_dev,
                          void* stream);
 
+/* Quest one-shot analogue (Section 5, "Query-aware baseline"): the mean query
+ * qbar of the window rows (the last W_eff = min(W, n) positions of the G query
+ * heads of each KV head; q_win as for snapkv_score) scores every page of `page`
+ * consecutive tokens of a sequence by the key bound
+ *   sum_i max(qbar_i * min_t k_ti, qbar_i * max_t k_ti)   (t over the page),
+ * an upper bound on qbar . k_t for every token of the page; the last page of a
+ * sequence may be short.  Every token's entry of `scores` (the layout of
+ * snapkv_score's output) is its page's bound, so role_alloc_select (pool_k 1,
+ * GLOBAL for Quest's plain page top-k, ties to the lower index keep whole pages
+ * in bound order) runs on it as on any score.
+ * d must be 64 or 128; 1 <= page <= 4096; W >= 1.  No workspace. */
+int quest_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k, int32_t W,
+                int32_t page, float* scores, void* stream);
+
 /* H2O accumulated attention mass (Section 2): s(t) = sum over the G query heads
  * of the KV head and every causal query position q >= t of p_t(q).
  *   q       bf16 prefill queries of every position: dense [L][b][Hq][n][d] or

@@ -17,6 +17,9 @@ matmul / sort as the only library steps:
                            Algorithm 1, the windowed-mass step).
 * ``h2o_score``         -- H2O accumulated mass s(t) = sum_q p_t(q) over every
                            causal query (Section 2).
+* ``quest_score``       -- the one-shot Quest analogue: page key-bounds against
+                           the window's mean query (Section 5, "Query-aware
+                           baseline").
 * ``maxpool1d``         -- the 1-D max-pool along the KV axis
                            (Algorithm 1, the pooling step; Section 4).
 * ``kept_count``,
@@ -150,6 +153,29 @@ def h2o_score(q: np.ndarray, k: np.ndarray, scale: float, row_block: int = 2048)
             P = attention_probs(q[g, r0:r1, :], k, np.arange(r0, r1), scale)
             s += P.sum(axis=0)
     return s
+
+
+def quest_score(q_win: np.ndarray, k: np.ndarray, W: int, page: int) -> np.ndarray:
+    """Quest one-shot analogue (Section 5, "Query-aware baseline"): the mean
+    query qbar of the window rows (the last W_eff = min(W, n) positions of all
+    G query heads of the KV head) scores every page of `page` consecutive
+    keys by Quest's key-bound, sum_i max(qbar_i * min_t k_ti, qbar_i *
+    max_t k_ti) over the page's tokens t, an upper bound on qbar . k_t for
+    every token of the page; every token gets its page's bound.  The last
+    page of a sequence may be short.  q_win is (G, W, d), k is (n, d)."""
+    k = np.asarray(k, dtype=np.float64)
+    n = k.shape[0]
+    out = np.zeros(n)
+    if n == 0:
+        return out
+    w_eff = min(W, n)
+    q = np.asarray(q_win, dtype=np.float64)[:, :w_eff, :]
+    qbar = q.reshape(-1, q.shape[-1]).mean(axis=0)
+    for p0 in range(0, n, page):
+        blk = k[p0:p0 + page]
+        lo, hi = blk.min(axis=0), blk.max(axis=0)
+        out[p0:p0 + page] = np.maximum(qbar * lo, qbar * hi).sum()
+    return out
 
 
 def maxpool1d(s: np.ndarray, kernel: int) -> np.ndarray:
@@ -361,6 +387,17 @@ def snapkv_batch(batch: Batch, q_win_bits, k_bits, W: int, pool_k: int,
         qw = bf16_to_f64(q_win_bits[l, s, h * batch.G:(h + 1) * batch.G, :, :])
         pre = snapkv_prepool(qw, k, W, scale)
         out[u] = (pre, maxpool1d(pre, pool_k) if pre.size else pre)
+    return out
+
+
+def quest_batch(batch: Batch, q_win_bits, k_bits, W: int, page: int, units: Iterable[int] | None = None):
+    """quest_score for every unit: {unit: per-token page bound}."""
+    out = {}
+    for u in (range(batch.n_units) if units is None else units):
+        l, s, h = batch.unit(u)
+        k = bf16_to_f64(batch.kv_rows(k_bits, u))
+        qw = bf16_to_f64(q_win_bits[l, s, h * batch.G:(h + 1) * batch.G])
+        out[u] = quest_score(qw, k, W, page)
     return out
 
 

@@ -83,6 +83,25 @@ struct SelectArgs {
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream);
 
+// Quest one-shot analogue ----------------------------------------------------
+
+struct QuestArgs {
+  int32_t L, b, G, Hkv, d, n_max;
+  int32_t varlen;
+  int64_t T;
+  const int32_t* cu_seqlens;
+  int32_t n_units;
+  int32_t W;                        // window rows per head averaged into the query
+  int32_t page;                     // tokens per page
+  const uint16_t* q;                // window queries (bf16 bits), SnapKV layout
+  int64_t q_layer, q_seq, q_head, q_tok;
+  const uint16_t* k;
+  int64_t k_layer, k_seq, k_head, k_tok;
+  float* scores;
+};
+
+cudaError_t launch_quest(const QuestArgs& a, cudaStream_t stream);
+
 // Compaction -----------------------------------------------------------------
 
 struct CompactArgs {

@@ -558,6 +558,53 @@ int h2o_score(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k, float
   return ROLEKV_OK;
 }
 
+int quest_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k, int32_t W,
+                int32_t page, float* scores, void* stream) {
+  BatchInfo bi;
+  int rc = check_batch(batch, &bi);
+  if (rc) return rc;
+  if (bi.d != 64 && bi.d != 128)
+    return fail(ROLEKV_ERR_UNSUPPORTED, "head dim %d (quest_score takes 64 or 128)", bi.d);
+  if (W < 1) return fail(ROLEKV_ERR_INVALID_ARG, "window W=%d must be >= 1", W);
+  if (page < 1 || page > 4096) return fail(ROLEKV_ERR_INVALID_ARG, "page=%d outside 1..4096", page);
+  if (scores == nullptr || (reinterpret_cast<uintptr_t>(scores) & 3u))
+    return fail(ROLEKV_ERR_INVALID_ARG, "scores must be a non-NULL, 4-byte aligned pointer");
+  if ((rc = check_tensor("q_win", q_win, bi.d, bi.Hq, false, false))) return rc;
+  if ((rc = check_tensor("k", k, bi.d, bi.Hkv, bi.varlen, false))) return rc;
+  if (bi.n_max == 0) return ROLEKV_OK;
+  QuestArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.L = bi.L;
+  a.b = bi.b;
+  a.G = bi.G;
+  a.Hkv = bi.Hkv;
+  a.d = bi.d;
+  a.n_max = bi.n_max;
+  a.varlen = bi.varlen;
+  a.T = bi.T;
+  a.cu_seqlens = batch->cu_seqlens_dev;
+  a.n_units = static_cast<int32_t>(bi.n_units);
+  a.W = W;
+  a.page = page;
+  a.q = static_cast<const uint16_t*>(q_win.ptr);
+  a.q_layer = q_win.s_layer;
+  a.q_seq = q_win.s_seq;
+  a.q_head = q_win.s_head;
+  a.q_tok = q_win.s_tok;
+  a.k = static_cast<const uint16_t*>(k.ptr);
+  a.k_layer = k.s_layer;
+  a.k_seq = k.s_seq;
+  a.k_head = k.s_head;
+  a.k_tok = k.s_tok;
+  a.scores = scores;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  stage_begin();
+  cudaError_t e = launch_quest(a, st);
+  if (e != cudaSuccess) return cuda_fail(e, "quest_score");
+  stage_mark(st);
+  return ROLEKV_OK;
+}
+
 int role_alloc_select(const rolekv_batch* batch, const float* scores, const uint8_t* roles,
                       const rolekv_select_params* params, int32_t pool_k, int32_t* keep_idx,
                       uint8_t* keep_mask, int32_t* kept_per_role, int32_t* status_dev,

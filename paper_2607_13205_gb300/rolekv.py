@@ -63,6 +63,9 @@ _SIGNATURES = [
     ("snapkv_score_noalloc", ctypes.c_int,
      [ctypes.POINTER(BatchDesc), Tensor, Tensor, ctypes.c_int32, ctypes.c_int32, ctypes.c_float,
       ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]),
+    ("quest_score", ctypes.c_int,
+     [ctypes.POINTER(BatchDesc), Tensor, Tensor, ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p,
+      ctypes.c_void_p]),
     ("h2o_score", ctypes.c_int,
      [ctypes.POINTER(BatchDesc), Tensor, Tensor, ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p,
       ctypes.c_size_t, ctypes.c_void_p, ctypes.c_void_p]),
@@ -228,6 +231,13 @@ def snapkv_score_noalloc(batch: Batch, q_win: torch.Tensor, k: torch.Tensor, W: 
     _check(lib().snapkv_score_noalloc(ctypes.byref(batch.desc), tensor_desc(q_win),
                                       tensor_desc(k, batch.varlen), W, pool_k, scale, _ptr(lse_win),
                                       _ptr(scores), _ptr(scores_prepool), _ptr(status), _stream(stream)))
+    return scores
+
+
+def quest_score(batch: Batch, q_win: torch.Tensor, k: torch.Tensor, W: int, page: int,
+                scores: torch.Tensor, stream=None) -> torch.Tensor:
+    _check(lib().quest_score(ctypes.byref(batch.desc), tensor_desc(q_win, False),
+                             tensor_desc(k, batch.varlen), W, page, _ptr(scores), _stream(stream)))
     return scores
 
 

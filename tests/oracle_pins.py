@@ -419,10 +419,40 @@ def pin_recency_floor(O, rng):
         assert per == [int((rl[0, kept] == x).sum()) for x in range(3)]
 
 
+def pin_quest_bound(O, rng):
+    """Quest page bound: with one-token pages it is the plain dot product of
+    the mean window query with each key; for any page it is at least every
+    member's dot product, reaches it when the page's keys are equal, does not
+    depend on the order of tokens inside a page, and the mean query is the
+    plain average of the G x W_eff window rows."""
+    G, W, d, n = 3, 5, 6, 37
+    qw = rng.standard_normal((G, W, d))
+    k = rng.standard_normal((n, d))
+    qbar = qw.reshape(-1, d).mean(axis=0)
+    assert np.allclose(O.quest_score(qw, k, W, 1), k @ qbar, rtol=1e-12, atol=1e-12)
+    for page in (2, 4, 16):
+        u = O.quest_score(qw, k, W, page)
+        dots = k @ qbar
+        for p0 in range(0, n, page):
+            assert np.all(u[p0:p0 + page] == u[p0])
+            assert u[p0] >= dots[p0:p0 + page].max() - 1e-12
+        perm = k.copy()
+        for p0 in range(0, n, page):
+            blk = perm[p0:p0 + page]
+            perm[p0:p0 + page] = blk[rng.permutation(blk.shape[0])]
+        assert np.allclose(O.quest_score(qw, perm, W, page), u, rtol=0, atol=1e-12)
+    same = np.repeat(rng.standard_normal((1, d)), 8, axis=0)
+    assert np.allclose(O.quest_score(qw, same, W, 8), same @ qbar, rtol=1e-12, atol=1e-12)
+    # a window longer than the sequence uses every position (W_eff = n)
+    short = rng.standard_normal((3, d))
+    qbar3 = qw[:, :3].reshape(-1, d).mean(axis=0)
+    assert np.allclose(O.quest_score(qw, short, W, 1), short @ qbar3, rtol=1e-12, atol=1e-12)
+
+
 ALL_PINS = [
     pin_rows_sum_to_one, pin_snapkv_total, pin_h2o_total, pin_uniform_closed_forms,
     pin_two_level_scale, pin_window_covering_is_h2o, pin_gqa_grouping, pin_maxpool,
     pin_kept_count, pin_quota_golden, pin_quota_waterlevel, pin_key_ban,
     pin_global_is_full_sort, pin_bruteforce_select, pin_compact, pin_varlen_matches_dense,
-    pin_fair_quotas, pin_recency_floor,
+    pin_fair_quotas, pin_recency_floor, pin_quest_bound,
 ]

@@ -192,3 +192,42 @@ def test_h2o_full_size():
         row = _unit_rows(ob, r["keep"], u, kept_off)
         check_index_sets(v.ob, 0, row, ref, v.roles, I.N_ROLES, I.PAPER_ALPHA, I.ROLE_KEY, 0.0, B)
         assert np.array_equal(_unit_rows(ob, ko_all, u, kept_off), O.compact_unit(v.k[0, 0, 0], row))
+
+
+def test_quest_long_full_size():
+    """Quest one-shot analogue on the long config (page 16, mean query of the
+    64-row window), then page top-k (GLOBAL, B=0.10) and compaction."""
+    w = I.WORKLOADS["long"]
+    B, page = w.budgets[0], 16
+    roles_np = I.workload_roles(w, 4)
+    K, V = I.make_kv(w, roles_np, 4, device=DEV)
+    qw = I.make_q_window(w, 4, device=DEV)
+    batch = lib_batch(w, DEV)
+    scores = torch.empty(batch.score_shape(), dtype=torch.float32, device=DEV)
+    R.quest_score(batch, qw, K, w.W, page, scores)
+    params = R.select_params(B, I.PAPER_ALPHA, 0.0, I.ROLE_KEY, policy=R.POLICY_GLOBAL)
+    keep = torch.empty(batch.kept_shape(B), dtype=torch.int32, device=DEV)
+    R.role_alloc_select(batch, scores, torch.as_tensor(roles_np, device=DEV), params, keep)
+    k_out = torch.empty(R.compact_shape(batch, B), dtype=torch.bfloat16, device=DEV)
+    v_out = torch.empty_like(k_out)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    R.kv_compact(batch, K, V, keep, B, k_out, v_out, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    ob = oracle_batch(w)
+    sc = scores.cpu().numpy().reshape(ob.n_units, -1)
+    assert np.all(np.isfinite(sc))
+    assert np.all(sc.reshape(ob.n_units, -1, page) == sc.reshape(ob.n_units, -1, page)[:, :, :1])
+    kp = keep.cpu().numpy().reshape(ob.n_units, -1)
+    Ks = O.kept_count(w.n, B)
+    assert kp.shape[1] == Ks and np.all(np.diff(kp, axis=1) > 0)
+    ko = I.bf16_bits(k_out).reshape(ob.n_units, Ks, -1)
+    for u in (0, 611, ob.n_units - 1):
+        v = UnitView(w, ob, u, K, V, roles_np, qw=qw)
+        ref = O.quest_score(O.bf16_to_f64(v.qw[0, 0]), O.bf16_to_f64(v.k[0, 0, 0]), w.W, page)
+        scale = np.abs(O.bf16_to_f64(v.qw[0, 0]).reshape(-1, w.d)[:w.G * w.W].mean(axis=0)).sum()
+        tol = 1e-5 * scale * np.abs(O.bf16_to_f64(v.k[0, 0, 0])).max() + 1e-4 * np.abs(ref)
+        assert np.all(np.abs(sc[u] - ref) <= tol)
+        check_index_sets(v.ob, 0, kp[u], ref, v.roles, I.N_ROLES, I.PAPER_ALPHA, I.ROLE_KEY, 0.0, B,
+                         policy=O.POLICY_GLOBAL)
+        assert np.array_equal(ko[u], O.compact_unit(v.k[0, 0, 0], kp[u]))

@@ -120,6 +120,60 @@ def test_h2o_score_matches_oracle(case):
             assert abs(ob.score_view(got, u).astype(np.float64).sum() - s.size * w.G) < 1e-3 * s.size * w.G
 
 
+# -------------------------------------------------------------------- quest
+
+QUEST_CASES = {
+    "tiny_d64_page16": (_w("tiny"), 16),
+    "g4_page16_ragged_tail": (_w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=3001), 16),
+    "page1_is_dot": (_w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=700), 1),
+    "page64_w64": (_w("long", L=1, b=1, Hq=8, Hkv=2, n=5000), 64),
+    "page5_g7": (_w("ragged", L=1, b=2, Hq=14, Hkv=2, n=2100, seqlens=None), 5),
+    "varlen_short_empty": (SNAPKV_CASES["varlen_short_empty"], 16),
+}
+
+
+def _quest_tol(ob, qb, kb, u, W, G):
+    """|qbar|_1 max|k|: the scale of the bound's rounding error."""
+    l, s, h = ob.unit(u)
+    k = O.bf16_to_f64(ob.kv_rows(kb, u))
+    if k.shape[0] == 0:
+        return 0.0
+    q = O.bf16_to_f64(qb[l, s, h * G:(h + 1) * G, :min(W, k.shape[0])]).reshape(-1, k.shape[1])
+    return float(np.abs(q.mean(axis=0)).sum() * np.abs(k).max())
+
+
+@pytest.mark.parametrize("case", list(QUEST_CASES))
+def test_quest_score_matches_oracle(case):
+    w, page = QUEST_CASES[case]
+    roles_np, K, V, qw = _snapkv_inputs(w, seed=6)
+    batch = lib_batch(w, DEV)
+    scores = torch.full(batch.score_shape(), float("nan"), dtype=torch.float32, device=DEV)
+    R.quest_score(batch, qw, K, w.W, page, scores)
+    torch.cuda.synchronize()
+    ob = oracle_batch(w)
+    qb, kb = I.bf16_bits(qw), I.bf16_bits(K)
+    ref = O.quest_batch(ob, qb, kb, w.W, page)
+    got_all = scores.cpu().numpy()
+    for u, r in ref.items():
+        got = ob.score_view(got_all, u).astype(np.float64)
+        tol = 1e-5 * _quest_tol(ob, qb, kb, u, w.W, w.G) + 1e-4 * np.abs(r)
+        assert np.all(np.abs(got - r) <= tol), f"{case} unit {u}"
+        for p0 in range(0, got.size, page):          # one bound per page
+            assert np.all(got[p0:p0 + page] == got[p0])
+    # page top-k: the GLOBAL selector on the bounds keeps whole pages
+    B = 0.10
+    params = R.select_params(B, I.PAPER_ALPHA, 0.0, I.ROLE_KEY, policy=R.POLICY_GLOBAL)
+    keep = torch.empty(batch.kept_shape(B), dtype=torch.int32, device=DEV)
+    R.role_alloc_select(batch, scores, torch.as_tensor(roles_np, device=DEV), params, keep)
+    torch.cuda.synchronize()
+    keep_np, cu = keep.cpu().numpy(), ob.kept_offsets(B)
+    for u, r in ref.items():
+        l, s, h = ob.unit(u)
+        row = keep_np[l, h, cu[s]:cu[s + 1]] if ob.varlen else keep_np.reshape(ob.n_units, -1)[u]
+        check_index_sets(ob, u, row, r, roles_np, I.N_ROLES, I.PAPER_ALPHA, I.ROLE_KEY, 0.0, B,
+                         policy=O.POLICY_GLOBAL)
+
+
 # ------------------------------------------------------------------ selection
 
 def _tied_scores(shape, seed):

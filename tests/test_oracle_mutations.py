@@ -198,6 +198,15 @@ def _m_floor_counts_whole_row(O):
                  ["select_batch"])
 
 
+def _m_quest_max_only(O):
+    _from_source(O, "np.maximum(qbar * lo, qbar * hi).sum()", "(qbar * hi).sum()", ["quest_score"])
+
+
+def _m_quest_window_start(O):
+    _from_source(O, "q = np.asarray(q_win, dtype=np.float64)[:, :w_eff, :]",
+                 "q = np.asarray(q_win, dtype=np.float64)", ["quest_score"])
+
+
 def _m_compact_off_by_one(O):
     orig = O.compact_unit
     O.compact_unit = lambda rows, idx: orig(rows, np.where(np.asarray(idx) >= 0, np.minimum(np.asarray(idx) + 1, rows.shape[0] - 1), -1))
@@ -208,7 +217,7 @@ MUTATIONS = [
     _m_mean_over_heads, _m_h2o_drops_heads, _m_pool_too_wide, _m_pool_one_sided,
     _m_round_not_ceil, _m_no_redistribution, _m_renormalise_all_buckets, _m_remainder_ties_high,
     _m_ties_to_high_index, _m_interleaved_gqa, _m_compact_off_by_one, _m_fair_uses_alpha,
-    _m_floor_outside_budget, _m_floor_counts_whole_row,
+    _m_floor_outside_budget, _m_floor_counts_whole_row, _m_quest_max_only, _m_quest_window_start,
 ]
 
 

@@ -20,6 +20,8 @@ matmul / sort as the only library steps:
 * ``quest_score``       -- the one-shot Quest analogue: page key-bounds against
                            the window's mean query (Section 5, "Query-aware
                            baseline").
+* ``decode_attention``  -- one decode step of attention through the compacted
+                           cache (Section 6).
 * ``maxpool1d``         -- the 1-D max-pool along the KV axis
                            (Algorithm 1, the pooling step; Section 4).
 * ``kept_count``,
@@ -176,6 +178,28 @@ def quest_score(q_win: np.ndarray, k: np.ndarray, W: int, page: int) -> np.ndarr
         lo, hi = blk.min(axis=0), blk.max(axis=0)
         out[p0:p0 + page] = np.maximum(qbar * lo, qbar * hi).sum()
     return out
+
+
+def decode_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, valid: np.ndarray,
+                     scale: float) -> np.ndarray:
+    """One decode step through a (compacted) cache: each of the G query rows
+    q (G, d) attends to the cache rows k, v (m, d) whose `valid` flag is set
+    (kept slots; the -1 padding of an infeasible budget is not), o_g =
+    sum_j softmax_j(scale q_g . k_j) v_j.  This is the step the compacted
+    cache exists for (Section 6: the 1-B memory and latency the masking
+    harness does not realise).  Returns (G, d); rows with no valid key give 0."""
+    q = np.asarray(q, dtype=np.float64)
+    k = np.asarray(k, dtype=np.float64)
+    v = np.asarray(v, dtype=np.float64)
+    valid = np.asarray(valid, dtype=bool)
+    out = np.zeros((q.shape[0], v.shape[1]))
+    if not valid.any():
+        return out
+    kk, vv = k[valid], v[valid]
+    logits = scale * (q @ kk.T)
+    m = logits.max(axis=1, keepdims=True)
+    e = np.exp(logits - m)
+    return (e / e.sum(axis=1, keepdims=True)) @ vv
 
 
 def maxpool1d(s: np.ndarray, kernel: int) -> np.ndarray:

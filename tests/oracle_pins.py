@@ -449,10 +449,38 @@ def pin_quest_bound(O, rng):
     assert np.allclose(O.quest_score(qw, short, W, 1), short @ qbar3, rtol=1e-12, atol=1e-12)
 
 
+def pin_decode_attention(O, rng):
+    """Decode attention: equal keys give the plain mean of the value rows; one
+    key far above the rest gives (nearly) its value row; the output is a
+    convex combination (inside the per-dim range of the values); row order
+    does not matter; rows flagged invalid are ignored whatever they hold; an
+    empty cache gives zero."""
+    G, m, d = 3, 20, 8
+    q = rng.standard_normal((G, d))
+    v = rng.standard_normal((m, d))
+    kc = np.repeat(rng.standard_normal((1, d)), m, axis=0)
+    ok = np.ones(m, dtype=bool)
+    assert np.allclose(O.decode_attention(q, kc, v, ok, 0.3), np.tile(v.mean(axis=0), (G, 1)),
+                       rtol=0, atol=1e-12)
+    k = rng.standard_normal((m, d))
+    k[7] = 50.0 * q[0] / np.linalg.norm(q[0])
+    o = O.decode_attention(q[:1], k, v, ok, 1.0)
+    assert np.allclose(o[0], v[7], atol=1e-6)
+    o = O.decode_attention(q, k, v, ok, 0.5)
+    assert np.all(o >= v.min(axis=0) - 1e-12) and np.all(o <= v.max(axis=0) + 1e-12)
+    perm = rng.permutation(m)
+    assert np.allclose(O.decode_attention(q, k[perm], v[perm], ok, 0.5), o, rtol=1e-12, atol=1e-12)
+    junk_k = np.vstack([k, 1e3 * rng.standard_normal((5, d))])
+    junk_v = np.vstack([v, 1e3 * rng.standard_normal((5, d))])
+    flags = np.concatenate([ok, np.zeros(5, dtype=bool)])
+    assert np.allclose(O.decode_attention(q, junk_k, junk_v, flags, 0.5), o, rtol=1e-12, atol=1e-12)
+    assert np.all(O.decode_attention(q, k, v, np.zeros(m, dtype=bool), 0.5) == 0)
+
+
 ALL_PINS = [
     pin_rows_sum_to_one, pin_snapkv_total, pin_h2o_total, pin_uniform_closed_forms,
     pin_two_level_scale, pin_window_covering_is_h2o, pin_gqa_grouping, pin_maxpool,
     pin_kept_count, pin_quota_golden, pin_quota_waterlevel, pin_key_ban,
     pin_global_is_full_sort, pin_bruteforce_select, pin_compact, pin_varlen_matches_dense,
-    pin_fair_quotas, pin_recency_floor, pin_quest_bound,
+    pin_fair_quotas, pin_recency_floor, pin_quest_bound, pin_decode_attention,
 ]

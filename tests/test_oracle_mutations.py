@@ -207,6 +207,14 @@ def _m_quest_window_start(O):
                  "q = np.asarray(q_win, dtype=np.float64)", ["quest_score"])
 
 
+def _m_decode_keeps_padding(O):
+    _from_source(O, "kk, vv = k[valid], v[valid]", "kk, vv = k, v", ["decode_attention"])
+
+
+def _m_decode_unnormalised(O):
+    _from_source(O, "return (e / e.sum(axis=1, keepdims=True)) @ vv", "return e @ vv", ["decode_attention"])
+
+
 def _m_compact_off_by_one(O):
     orig = O.compact_unit
     O.compact_unit = lambda rows, idx: orig(rows, np.where(np.asarray(idx) >= 0, np.minimum(np.asarray(idx) + 1, rows.shape[0] - 1), -1))
@@ -218,6 +226,7 @@ MUTATIONS = [
     _m_round_not_ceil, _m_no_redistribution, _m_renormalise_all_buckets, _m_remainder_ties_high,
     _m_ties_to_high_index, _m_interleaved_gqa, _m_compact_off_by_one, _m_fair_uses_alpha,
     _m_floor_outside_budget, _m_floor_counts_whole_row, _m_quest_max_only, _m_quest_window_start,
+    _m_decode_keeps_padding, _m_decode_unnormalised,
 ]
 
 

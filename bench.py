@@ -334,6 +334,8 @@ def run_gpu(args):
         result["single_pass"] = run_single_pass(args, batch, params, w, B, qw, K, V, roles, scores,
                                                 keep, k_out, v_out, ws, status, stream, world,
                                                 seq_tokens)
+    if not h2o and not args.no_decode:
+        result["decode"] = run_decode(args, batch, w, B, K, V, keep, k_out, v_out, stream, world, peaks)
     if not args.no_e2e:
         result["e2e"] = run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep,
                                 k_out, v_out, status, stream, world, seq_tokens)
@@ -422,6 +424,50 @@ def run_single_pass(args, batch, params, w, B, qw, K, V, roles, scores, keep, k_
     return {"value": world * seq_tokens * steps / (total / 1e3), "unit": UNIT,
             "ms_per_step": total / steps, "score_ms": score_ms, "steps": steps,
             "lse": "window normalisers supplied by the caller (computed once, untimed)"}
+
+
+def run_decode(args, batch, w, B, K, V, keep, k_out, v_out, stream, world, peaks):
+    """One decode step of attention (a new token per sequence, every head)
+    through the compacted cache the step just built, and through the full
+    cache, each timed over the same number of iterations."""
+    import torch
+
+    from paper_2607_13205_gb300 import inputs as I
+    from paper_2607_13205_gb300 import rolekv as R
+
+    qd = I.make_q_decode(w, 11, device=K.device)
+    out = torch.empty((w.L, w.b, w.Hq, w.d), dtype=torch.float32, device=K.device)
+    ws_c = R.decode_workspace(batch, B, device=K.device)
+    ws_f = R.decode_workspace(batch, 1.0, device=K.device)
+    units = w.L * w.b * w.Hkv
+    rows_c = (sum(math.ceil(B * x) for x in w.seqlens) if w.varlen else w.b * math.ceil(B * w.n)) * w.L * w.Hkv
+    rows_f = (sum(w.seqlens) if w.varlen else w.b * w.n) * w.L * w.Hkv
+    del units
+
+    def timed(fn, reps):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        barrier(world)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return max_over_ranks(e0.elapsed_time(e1) / reps, world)
+
+    reps = max(3, args.steps)
+    t_c = timed(lambda: R.decode_attention(batch, qd, k_out, v_out, keep, B, out, ws=ws_c, stream=stream), reps)
+    t_f = timed(lambda: R.decode_attention(batch, qd, K, V, None, 1.0, out, compacted=False, ws=ws_f,
+                                           stream=stream), reps)
+    by_c = rows_c * w.d * 2 * 2 + rows_c * 4
+    by_f = rows_f * w.d * 2 * 2
+    return {"compacted_ms": t_c, "full_ms": t_f, "speedup": t_f / t_c,
+            "compacted_hbm_frac": by_c / (t_c / 1e3) / 1e9 / peaks["hbm_gbs"],
+            "full_hbm_frac": by_f / (t_f / 1e3) / 1e9 / peaks["hbm_gbs"],
+            "bytes": {"compacted": by_c, "full": by_f},
+            "what": "one decode token per sequence, all heads; full = budget 1, no index"}
 
 
 def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_out, v_out, status,
@@ -625,6 +671,8 @@ def main(argv=None):
     ap.add_argument("--no-single-pass", action="store_true",
                     help="skip the step with caller-supplied window normalisers")
     ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--no-decode", action="store_true",
+                    help="skip the decode-step timing through the compacted and the full cache")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-units", type=int, default=2)

@@ -205,6 +205,30 @@ int snapkv_score_noalloc(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_
 int quest_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k, int32_t W,
                 int32_t page, float* scores, void* stream);
 
+/* One decode step of attention through a cache of kept rows (Section 6: the
+ * compacted cache realises the 1-B memory and decode-time reduction).  For
+ * every (layer, sequence, KV head) and each of its G query heads,
+ *   out_g = sum_j softmax_j(scale * q_g . k_j) v_j
+ * over the unit's rows j < ceil(budget * n) of k_cache / v_cache, skipping the
+ * rows whose keep_idx entry is -1 (the padding of an infeasible budget).
+ *   q        bf16 decode queries, one token per sequence: [L][b][Hq][d]
+ *            (s_tok is ignored).
+ *   k_cache, v_cache  bf16 cache rows: kv_compact's output (dense
+ *            [L][b][Hkv][K][d], varlen [L][Hkv][Ktot][d]: token index =
+ *            kept rows of the earlier sequences + j), or, with budget 1 and
+ *            keep_idx NULL, the full cache in its own layout (varlen
+ *            [L][T][Hkv][d]).
+ *   keep_idx the kept index rows role_alloc_select wrote, or NULL (all valid).
+ *   scale    <= 0: 1/sqrt(d).
+ *   out      fp32 [L][b][Hq][d], contiguous.
+ *   workspace  rolekv_decode_workspace_size() bytes (partials of the split
+ *            rows), caller-owned, no initialisation needed.
+ * d must be 64 or 128 and G <= 8; a unit with no valid row gives zeros. */
+int rolekv_decode_workspace_size(const rolekv_batch* batch, float budget, size_t* bytes);
+int decode_attention(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k_cache,
+                     rolekv_tensor v_cache, const int32_t* keep_idx, float budget, float scale,
+                     float* out, void* workspace, size_t workspace_bytes, void* stream);
+
 /* H2O accumulated attention mass (Section 2): s(t) = sum over the G query heads
  * of the KV head and every causal query position q >= t of p_t(q).
  *   q       bf16 prefill queries of every position: dense [L][b][Hq][n][d] or

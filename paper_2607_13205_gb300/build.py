@@ -19,7 +19,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(ROOT, "_build")
 LIB_PATH = os.path.join(PKG_DIR, "librolekv.so")
 
-SOURCES = ["rolekv_api.cu", "attn_score.cu", "select.cu", "compact.cu", "quest.cu"]
+SOURCES = ["rolekv_api.cu", "attn_score.cu", "select.cu", "compact.cu", "quest.cu", "decode.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

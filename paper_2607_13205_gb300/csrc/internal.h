@@ -102,6 +102,33 @@ struct QuestArgs {
 
 cudaError_t launch_quest(const QuestArgs& a, cudaStream_t stream);
 
+// Decode attention through the (compacted) cache -----------------------------
+
+struct DecodeArgs {
+  int32_t L, b, G, Hkv, d, n_max;
+  int32_t varlen;
+  const int32_t* cu_seqlens;
+  int32_t n_units;
+  int64_t budget_fx;                // rows of a sequence: kept_slots(n, budget_fx)
+  int64_t Ktot;                     // packed rows per (layer, head), varlen
+  int32_t K_dense;                  // rows per unit, dense
+  const uint16_t* q;                // decode queries [L][b][Hq][d] (strides below)
+  int64_t q_layer, q_seq, q_head;
+  const uint16_t* k;
+  int64_t k_layer, k_seq, k_head, k_tok;
+  const uint16_t* v;
+  int64_t v_layer, v_seq, v_head, v_tok;
+  const int32_t* keep_idx;          // -1 marks an empty slot; NULL: every row valid
+  float c1;                         // scale * log2(e)
+  int32_t rows_per_split;
+  int32_t n_splits;
+  float* part;                      // [unit][split][G][d + 2]: o (unnormalised), max2, sum
+  float* out;                       // fp32 outputs
+  int64_t o_layer, o_seq, o_head;
+};
+
+cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
+
 // Compaction -----------------------------------------------------------------
 
 struct CompactArgs {

@@ -635,6 +635,118 @@ int role_alloc_select(const rolekv_batch* batch, const float* scores, const uint
   return ROLEKV_OK;
 }
 
+namespace {
+constexpr int kDecodeRowsPerSplit = 512;
+
+// Rows of the largest sequence and the packed row total at this budget.
+void decode_rows(const BatchInfo& bi, const rolekv_batch* bt, int64_t bfx, int64_t* m_max,
+                 int64_t* total) {
+  *m_max = 0;
+  *total = 0;
+  if (bi.varlen) {
+    for (int s = 0; s < bi.b; ++s) {
+      const int64_t m = kept_slots(bt->seqlens_host[s], bfx);
+      *m_max = m > *m_max ? m : *m_max;
+      *total += m;
+    }
+  } else {
+    *m_max = kept_slots(bi.n_max, bfx);
+    *total = *m_max * bi.b;
+  }
+}
+
+size_t decode_ws_bytes(const BatchInfo& bi, int64_t m_max) {
+  const int64_t splits = (m_max + kDecodeRowsPerSplit - 1) / kDecodeRowsPerSplit;
+  return static_cast<size_t>(bi.n_units) * static_cast<size_t>(splits > 0 ? splits : 1) * bi.G *
+         (bi.d + 2) * sizeof(float);
+}
+}  // namespace
+
+int rolekv_decode_workspace_size(const rolekv_batch* batch, float budget, size_t* bytes) {
+  BatchInfo bi;
+  int rc = check_batch(batch, &bi);
+  if (rc) return rc;
+  if (bytes == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "bytes is NULL");
+  if (!(budget > 0.f) || budget > 1.f)
+    return fail(ROLEKV_ERR_INVALID_ARG, "budget %g outside (0, 1]", static_cast<double>(budget));
+  int64_t m_max, total;
+  decode_rows(bi, batch, to_fixed(budget), &m_max, &total);
+  *bytes = decode_ws_bytes(bi, m_max);
+  return ROLEKV_OK;
+}
+
+int decode_attention(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k_cache,
+                     rolekv_tensor v_cache, const int32_t* keep_idx, float budget, float scale,
+                     float* out, void* workspace, size_t workspace_bytes, void* stream) {
+  BatchInfo bi;
+  int rc = check_batch(batch, &bi);
+  if (rc) return rc;
+  if (bi.d != 64 && bi.d != 128)
+    return fail(ROLEKV_ERR_UNSUPPORTED, "head dim %d (decode_attention takes 64 or 128)", bi.d);
+  if (bi.G > 8) return fail(ROLEKV_ERR_UNSUPPORTED, "G=%d query heads per KV head (at most 8)", bi.G);
+  if (!(budget > 0.f) || budget > 1.f)
+    return fail(ROLEKV_ERR_INVALID_ARG, "budget %g outside (0, 1]", static_cast<double>(budget));
+  if (out == nullptr || (reinterpret_cast<uintptr_t>(out) & 15u))
+    return fail(ROLEKV_ERR_INVALID_ARG, "out must be a non-NULL, 16-byte aligned pointer");
+  if (q.ptr == nullptr || (reinterpret_cast<uintptr_t>(q.ptr) & 15u) || q.s_head < bi.d ||
+      q.s_layer < 0 || q.s_seq < 0 || (q.s_head % 8) || (q.s_seq % 8) || (q.s_layer % 8))
+    return fail(ROLEKV_ERR_INVALID_ARG, "q: NULL, misaligned or bad strides");
+  if ((rc = check_tensor("k_cache", k_cache, bi.d, bi.Hkv, bi.varlen, false))) return rc;
+  if ((rc = check_tensor("v_cache", v_cache, bi.d, bi.Hkv, bi.varlen, false))) return rc;
+  const int64_t bfx = to_fixed(budget);
+  int64_t m_max, total;
+  decode_rows(bi, batch, bfx, &m_max, &total);
+  const size_t need = decode_ws_bytes(bi, m_max);
+  if (workspace == nullptr || workspace_bytes < need)
+    return fail(ROLEKV_ERR_WORKSPACE, "workspace of %zu bytes, %zu needed", workspace_bytes, need);
+  if (reinterpret_cast<uintptr_t>(workspace) & 255u)
+    return fail(ROLEKV_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+  if (m_max == 0) return ROLEKV_OK;
+  DecodeArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.L = bi.L;
+  a.b = bi.b;
+  a.G = bi.G;
+  a.Hkv = bi.Hkv;
+  a.d = bi.d;
+  a.n_max = bi.n_max;
+  a.varlen = bi.varlen;
+  a.cu_seqlens = batch->cu_seqlens_dev;
+  a.n_units = static_cast<int32_t>(bi.n_units);
+  a.budget_fx = bfx;
+  a.Ktot = bi.varlen ? total : 0;
+  a.K_dense = bi.varlen ? 0 : static_cast<int32_t>(m_max);
+  a.q = static_cast<const uint16_t*>(q.ptr);
+  a.q_layer = q.s_layer;
+  a.q_seq = q.s_seq;
+  a.q_head = q.s_head;
+  a.k = static_cast<const uint16_t*>(k_cache.ptr);
+  a.k_layer = k_cache.s_layer;
+  a.k_seq = k_cache.s_seq;
+  a.k_head = k_cache.s_head;
+  a.k_tok = k_cache.s_tok;
+  a.v = static_cast<const uint16_t*>(v_cache.ptr);
+  a.v_layer = v_cache.s_layer;
+  a.v_seq = v_cache.s_seq;
+  a.v_head = v_cache.s_head;
+  a.v_tok = v_cache.s_tok;
+  a.keep_idx = keep_idx;
+  a.c1 = (scale > 0.f ? scale : 1.0f / std::sqrt(static_cast<float>(bi.d))) * 1.4426950408889634f;
+  a.rows_per_split = kDecodeRowsPerSplit;
+  a.n_splits = static_cast<int32_t>((m_max + kDecodeRowsPerSplit - 1) / kDecodeRowsPerSplit);
+  a.part = static_cast<float*>(workspace);
+  a.out = out;
+  a.o_seq = static_cast<int64_t>(bi.Hq) * bi.d;
+  a.o_layer = a.o_seq * bi.b;
+  a.o_head = bi.d;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  stage_begin();
+  cudaError_t e = launch_decode(a, st);
+  if (e != cudaSuccess) return cuda_fail(e, "decode_attention");
+  stage_mark(st);
+  return ROLEKV_OK;
+}
+
 int kv_compact(const rolekv_batch* batch, rolekv_tensor k, rolekv_tensor v,
                const int32_t* keep_idx, float budget, void* k_out, void* v_out,
                int32_t* status_dev, void* stream) {

@@ -209,6 +209,15 @@ def make_q_window(w: Workload, seed: int = 0, device="cpu") -> torch.Tensor:
     return z.to(torch.bfloat16)
 
 
+def make_q_decode(w: Workload, seed: int = 0, device="cpu") -> torch.Tensor:
+    """One decode query per sequence and head [L][b][Hq][d] (bf16), drawn like
+    the window queries."""
+    u = _directions(w, seed, device)
+    z = torch.randn(w.L, w.b, w.Hq, w.d, generator=_gen(device, seed, 5), device=device)
+    z += QUERY_SHIFT * u.repeat_interleave(w.G, dim=1)[:, None, :, :]
+    return z.to(torch.bfloat16)
+
+
 def make_q_full(w: Workload, seed: int = 0, device="cpu") -> torch.Tensor:
     """All prefill queries (H2O): dense [L][b][Hq][n][d] or packed [L][T][Hq][d]."""
     u = _directions(w, seed, device)

@@ -66,6 +66,11 @@ _SIGNATURES = [
     ("quest_score", ctypes.c_int,
      [ctypes.POINTER(BatchDesc), Tensor, Tensor, ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p,
       ctypes.c_void_p]),
+    ("rolekv_decode_workspace_size", ctypes.c_int,
+     [ctypes.POINTER(BatchDesc), ctypes.c_float, ctypes.POINTER(ctypes.c_size_t)]),
+    ("decode_attention", ctypes.c_int,
+     [ctypes.POINTER(BatchDesc), Tensor, Tensor, Tensor, ctypes.c_void_p, ctypes.c_float,
+      ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]),
     ("h2o_score", ctypes.c_int,
      [ctypes.POINTER(BatchDesc), Tensor, Tensor, ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p,
       ctypes.c_size_t, ctypes.c_void_p, ctypes.c_void_p]),
@@ -239,6 +244,38 @@ def quest_score(batch: Batch, q_win: torch.Tensor, k: torch.Tensor, W: int, page
     _check(lib().quest_score(ctypes.byref(batch.desc), tensor_desc(q_win, False),
                              tensor_desc(k, batch.varlen), W, page, _ptr(scores), _stream(stream)))
     return scores
+
+
+def decode_workspace(batch: Batch, budget: float, device="cuda") -> torch.Tensor:
+    out = ctypes.c_size_t(0)
+    _check(lib().rolekv_decode_workspace_size(ctypes.byref(batch.desc), budget, ctypes.byref(out)))
+    return torch.empty(max(int(out.value), 256), dtype=torch.uint8, device=device)
+
+
+def cache_desc(t: torch.Tensor, batch: Batch, compacted: bool) -> Tensor:
+    """Strides of a cache tensor: kv_compact's output (compacted=True:
+    dense [L][b][Hkv][K][d], varlen [L][Hkv][Ktot][d]) or an uncompacted K/V
+    in the library's own layouts."""
+    if compacted and batch.varlen:
+        return tensor_desc(t.transpose(1, 2), True)
+    return tensor_desc(t, batch.varlen)
+
+
+def decode_attention(batch: Batch, q: torch.Tensor, k_cache: torch.Tensor, v_cache: torch.Tensor,
+                     keep_idx: Optional[torch.Tensor], budget: float, out: torch.Tensor,
+                     compacted: bool = True, scale: float = 0.0, ws: Optional[torch.Tensor] = None,
+                     stream=None) -> torch.Tensor:
+    """q bf16 [L][b][Hq][d] -> out fp32 [L][b][Hq][d]."""
+    if ws is None:
+        ws = decode_workspace(batch, budget, device=q.device)
+    if q.dtype != torch.bfloat16 or q.dim() != 4 or q.stride(-1) != 1:
+        raise ValueError("q is a bf16 [L][b][Hq][d] tensor with a contiguous last axis")
+    sl, ss, sh, _ = q.stride()
+    qd = Tensor(q.data_ptr(), sl, ss, sh, q.shape[-1])
+    _check(lib().decode_attention(ctypes.byref(batch.desc), qd, cache_desc(k_cache, batch, compacted),
+                                  cache_desc(v_cache, batch, compacted), _ptr(keep_idx), budget, scale,
+                                  _ptr(out), _ptr(ws), ws.numel(), _stream(stream)))
+    return out
 
 
 def h2o_score(batch: Batch, q: torch.Tensor, k: torch.Tensor, scores: torch.Tensor, scale: float = 0.0,

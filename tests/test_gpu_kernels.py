@@ -174,6 +174,89 @@ def test_quest_score_matches_oracle(case):
                          policy=O.POLICY_GLOBAL)
 
 
+# ------------------------------------------------------------------- decode
+
+DECODE_CASES = {
+    # name: (workload, budget, policy, ban_mask)
+    "g4_b10": (_w("llama8b", L=2, b=2, Hq=8, Hkv=2, n=3001), 0.10, 0, 0),
+    "d64": (_w("tiny", b=2), 0.30, 0, 0),
+    "g7_varlen": (_w("ragged", L=1, b=3, Hq=14, Hkv=2, n=1500, seqlens=(1500, 31, 640)), 0.10, 0, 0),
+    "varlen_empty_infeasible": (SNAPKV_CASES["varlen_short_empty"], 0.60, R.POLICY_GLOBAL,
+                                ~(1 << I.ROLE_VALUE) & 0xF),
+}
+
+
+def _decode_ref(ob, w, qd_bits, kc, vc, valid_of):
+    out = {}
+    for u in range(ob.n_units):
+        l, s, h = ob.unit(u)
+        q = O.bf16_to_f64(qd_bits[l, s, h * w.G:(h + 1) * w.G])
+        k, v, ok = kc(u), vc(u), valid_of(u)
+        out[u] = O.decode_attention(q, O.bf16_to_f64(k), O.bf16_to_f64(v), ok, 1.0 / np.sqrt(w.d))
+    return out
+
+
+def _check_decode(ob, w, got, ref, vmax):
+    g = got.cpu().numpy()
+    for u, r in ref.items():
+        l, s, h = ob.unit(u)
+        o = g[l, s, h * w.G:(h + 1) * w.G].astype(np.float64)
+        assert np.all(np.abs(o - r) <= 1e-3 * np.abs(r) + 1e-4 * vmax), f"unit {u}"
+
+
+@pytest.mark.parametrize("case", list(DECODE_CASES))
+def test_decode_attention_compacted(case):
+    """Score -> select -> compact -> one decode step through the compacted
+    cache, against the oracle on the compacted rows (-1 slots masked)."""
+    w, B, policy, ban = DECODE_CASES[case]
+    roles_np, K, V, qw = _snapkv_inputs(w, seed=7)
+    batch = lib_batch(w, DEV)
+    scores = torch.empty(batch.score_shape(), dtype=torch.float32, device=DEV)
+    R.snapkv_score(batch, qw, K, w.W, w.pool_k, scores)
+    keep = torch.empty(batch.kept_shape(B), dtype=torch.int32, device=DEV)
+    R.role_alloc_select(batch, scores, torch.as_tensor(roles_np, device=DEV),
+                        R.select_params(B, I.PAPER_ALPHA, 0.0, I.ROLE_KEY, policy=policy, ban_mask=ban),
+                        keep)
+    kc = torch.empty(R.compact_shape(batch, B), dtype=torch.bfloat16, device=DEV)
+    vc = torch.empty_like(kc)
+    R.kv_compact(batch, K, V, keep, B, kc, vc)
+    qd = I.make_q_decode(w, 7, device=DEV)
+    out = torch.full((w.L, w.b, w.Hq, w.d), float("nan"), dtype=torch.float32, device=DEV)
+    for _ in range(2):                               # the workspace holds no state
+        R.decode_attention(batch, qd, kc, vc, keep, B, out)
+    torch.cuda.synchronize()
+    ob = oracle_batch(w)
+    kb, vb, kp = I.bf16_bits(kc), I.bf16_bits(vc), keep.cpu().numpy()
+    cu = ob.kept_offsets(B)
+
+    def rows(arr, u):
+        l, s, h = ob.unit(u)
+        return arr[l, h, cu[s]:cu[s + 1]] if ob.varlen else arr.reshape((ob.n_units, -1) + arr.shape[4:])[u]
+    ref = _decode_ref(ob, w, I.bf16_bits(qd), lambda u: rows(kb, u), lambda u: rows(vb, u),
+                      lambda u: rows(kp, u) >= 0)
+    _check_decode(ob, w, out, ref, float(V.float().abs().max()))
+    if case == "varlen_empty_infeasible":
+        assert any((rows(kp, u) < 0).any() for u in range(ob.n_units))   # padding was exercised
+
+
+@pytest.mark.parametrize("varlen", [False, True])
+def test_decode_attention_full_cache(varlen):
+    """Budget 1 and no index: attention over every cached token, in the
+    uncompacted K/V layouts."""
+    w = (SNAPKV_CASES["varlen_g7"] if varlen else _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=2000))
+    roles_np, K, V, _ = _snapkv_inputs(w, seed=8)
+    batch = lib_batch(w, DEV)
+    qd = I.make_q_decode(w, 8, device=DEV)
+    out = torch.empty((w.L, w.b, w.Hq, w.d), dtype=torch.float32, device=DEV)
+    R.decode_attention(batch, qd, K, V, None, 1.0, out, compacted=False)
+    torch.cuda.synchronize()
+    ob = oracle_batch(w)
+    kb, vb = I.bf16_bits(K), I.bf16_bits(V)
+    ref = _decode_ref(ob, w, I.bf16_bits(qd), lambda u: ob.kv_rows(kb, u), lambda u: ob.kv_rows(vb, u),
+                      lambda u: np.ones(ob.kv_rows(kb, u).shape[0], dtype=bool))
+    _check_decode(ob, w, out, ref, float(V.float().abs().max()))
+
+
 # ------------------------------------------------------------------ selection
 
 def _tied_scores(shape, seed):

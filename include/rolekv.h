@@ -223,11 +223,13 @@ int quest_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k,
  *   out      fp32 [L][b][Hq][d], contiguous.
  *   workspace  rolekv_decode_workspace_size() bytes (partials of the split
  *            rows), caller-owned, no initialisation needed.
+ *   status_dev optional int32 status word (ROLEKV_STATUS_TIMEOUT).
  * d must be 64 or 128 and G <= 8; a unit with no valid row gives zeros. */
 int rolekv_decode_workspace_size(const rolekv_batch* batch, float budget, size_t* bytes);
 int decode_attention(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k_cache,
                      rolekv_tensor v_cache, const int32_t* keep_idx, float budget, float scale,
-                     float* out, void* workspace, size_t workspace_bytes, void* stream);
+                     float* out, void* workspace, size_t workspace_bytes, int32_t* status_dev,
+                     void* stream);
 
 /* H2O accumulated attention mass (Section 2): s(t) = sum over the G query heads
  * of the KV head and every causal query position q >= t of p_t(q).

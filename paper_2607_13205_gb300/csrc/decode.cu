@@ -4,13 +4,16 @@
 //   o_g = sum_j softmax_j(scale q_g . k_j) v_j
 // over the unit's cache rows (the kept slots; -1 slots of an infeasible budget
 // are skipped; with budget 1 and no index the full cache).  Memory-bound: the
-// cache rows are read once.  Split-K: CTA (unit, split) takes 512 rows; each of
-// its four warps takes its own batches of 8 rows (4 when G > 4) for all G
-// query heads, lanes over the head dimension: the batch's loads go out
-// together, the G x rows dot products are reduced across the warp, and an
-// online softmax per head keeps (max, sum, unnormalised output) in log2
-// units.  The warps merge through shared memory; a second launch merges the
-// splits of each (unit, head).
+// cache rows are read once.  Split-K: CTA (unit, split) takes 512 rows.  A
+// producer warp streams them into four shared-memory stages of 32 K rows and
+// 32 V rows with bulk copies (one per stage when a unit's rows are
+// contiguous, one per row otherwise), so the bytes in flight do not depend on
+// registers; each of four consumer warps takes 8 rows of every stage for all
+// G query heads, lanes over the head dimension: the G x rows dot products are
+// reduced across the warp and an online softmax per head keeps (max, sum,
+// unnormalised output) in log2 units.  Every wait is a bounded mbarrier wait.
+// The warps merge through shared memory; a second launch merges the splits of
+// each (unit, head).
 #include <cuda_runtime.h>
 
 #include <cmath>
@@ -64,11 +67,19 @@ __device__ __forceinline__ int64_t kept_prefix(const DecodeArgs& a, int s) {
   return part;
 }
 
-constexpr int kDecWarps = 4;       // warps per CTA, each on its own rows
+constexpr int kDecWarps = 4;       // consumer warps per CTA
+constexpr int kStages = 4;         // shared-memory stages of cache rows
+constexpr int kStageRows = 32;     // rows per stage (8 per consumer warp)
+constexpr int kDecThreads = (kDecWarps + 1) * 32;   // + one producer warp
+
+__host__ __device__ constexpr int decode_smem_bytes(int d) { return 2 * kStages * kStageRows * d * 2; }
 
 template <int DPL, int GM>
-__global__ void __launch_bounds__(kDecWarps * 32) decode_partial_kernel(const DecodeArgs a) {
+__global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const DecodeArgs a) {
   constexpr int RB = GM <= 4 ? kRowBatch : kRowBatch / 2;   // rows per batch (registers)
+  extern __shared__ __align__(128) uint8_t stage_mem[];     // K stages, then V stages
+  __shared__ uint64_t full_bar[kStages], empty_bar[kStages];
+  __shared__ int abort_flag;
   __shared__ float red[kDecWarps][GM][2];                   // per-warp (max2, sum) per head
   __shared__ float racc[kDecWarps][GM][128];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -91,22 +102,22 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_partial_kernel(const De
   const int r0 = split * a.rows_per_split;
   if (r0 >= m) return;                              // (uniform: no partial is read)
   const int r1 = (m - r0 < a.rows_per_split) ? m : r0 + a.rows_per_split;
-  const int d0 = lane * DPL;
+  const int nst = (r1 - r0 + kStageRows - 1) / kStageRows;
+  const int rowbytes = a.d * 2;
+  const int64_t kb = l * a.k_layer + (a.varlen ? row0 * a.k_tok : s * a.k_seq) + h * a.k_head;
+  const int64_t vb = l * a.v_layer + (a.varlen ? row0 * a.v_tok : s * a.v_seq) + h * a.v_head;
+  uint8_t* ks = stage_mem;
+  uint8_t* vs = stage_mem + kStages * kStageRows * rowbytes;
 
-  // the G query heads' DPL dims, pre-scaled by scale * log2(e)
-  float q[GM][DPL];
-#pragma unroll
-  for (int g = 0; g < GM; ++g) {
-    const uint16_t* qp = a.q + l * a.q_layer + s * a.q_seq + static_cast<int64_t>(h * G + (g < G ? g : 0)) * a.q_head + d0;
-#pragma unroll
-    for (int i = 0; i < DPL; ++i) q[g][i] = g < G ? bf16f(qp[i]) * a.c1 : 0.f;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kStages; ++i) {
+      mbar_init(&full_bar[i], 1);
+      mbar_init(&empty_bar[i], kDecWarps);
+    }
+    abort_flag = 0;
+    fence_mbar_init();
   }
-  const int64_t kb = l * a.k_layer + (a.varlen ? row0 * a.k_tok : s * a.k_seq) + h * a.k_head + d0;
-  const int64_t vb = l * a.v_layer + (a.varlen ? row0 * a.v_tok : s * a.v_seq) + h * a.v_head + d0;
-  const int32_t* idx = nullptr;
-  if (a.keep_idx != nullptr)
-    idx = a.keep_idx + (a.varlen ? (static_cast<int64_t>(l) * a.Hkv + h) * a.Ktot + row0
-                                 : static_cast<int64_t>(u) * a.K_dense);
+  __syncthreads();
 
   float mx[GM], sum[GM], acc[GM][DPL];
 #pragma unroll
@@ -116,107 +127,172 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_partial_kernel(const De
 #pragma unroll
     for (int i = 0; i < DPL; ++i) acc[g][i] = 0.f;
   }
-  // warp w takes the batches w, w + kDecWarps, ... of the split's rows
-  for (int rb = r0 + warp * RB; rb < r1; rb += kDecWarps * RB) {
-    // all loads first and unconditional (rows past the end re-read the last
-    // row and are masked below), so the batch's loads are in flight together
-    RawDims<DPL> kraw[RB], vraw[RB];
-#pragma unroll
-    for (int j = 0; j < RB; ++j) {
-      const int r = (rb + j < r1) ? rb + j : r1 - 1;
-      kraw[j] = load_raw<DPL>(a.k + kb + r * a.k_tok);
-      vraw[j] = load_raw<DPL>(a.v + vb + r * a.v_tok);
-    }
-    bool ok[RB];
-#pragma unroll
-    for (int j = 0; j < RB; ++j) {
-      const int r = (rb + j < r1) ? rb + j : r1 - 1;
-      ok[j] = (rb + j < r1) && (idx == nullptr || __ldg(idx + r) >= 0);
-    }
-    float sc[GM][RB];
-#pragma unroll
-    for (int j = 0; j < RB; ++j) {
-      float kr[DPL];
-      unpack<DPL>(kraw[j], kr);
-#pragma unroll
-      for (int g = 0; g < GM; ++g) {
-        float t = 0.f;
-#pragma unroll
-        for (int i = 0; i < DPL; ++i) t = fmaf(q[g][i], kr[i], t);
-        sc[g][j] = t;
+
+  if (warp == kDecWarps) {
+    // ---------------------------------------------------------- producer
+    const bool kc = a.k_tok == a.d, vc = a.v_tok == a.d;   // rows contiguous
+    int issued = 0;
+    for (int st = 0; st < nst; ++st) {
+      const int slot = st % kStages;
+      bool ok = true;
+      if (lane == 0) ok = mbar_wait(&empty_bar[slot], ((st / kStages) & 1) ^ 1, &abort_flag, a.status);
+      if (!__shfl_sync(0xffffffffu, static_cast<int>(ok), 0)) break;
+      const int rs = r0 + st * kStageRows;
+      const int nr = (r1 - rs < kStageRows) ? r1 - rs : kStageRows;
+      if (lane == 0) mbar_arrive_expect_tx(&full_bar[slot], static_cast<uint32_t>(2 * nr * rowbytes));
+      __syncwarp();
+      uint8_t* kd = ks + slot * kStageRows * rowbytes;
+      uint8_t* vd = vs + slot * kStageRows * rowbytes;
+      if (kc) {
+        if (lane == 0) bulk_copy_g2s(kd, a.k + kb + static_cast<int64_t>(rs) * a.k_tok, nr * rowbytes, &full_bar[slot]);
+      } else if (lane < nr) {
+        bulk_copy_g2s(kd + lane * rowbytes, a.k + kb + static_cast<int64_t>(rs + lane) * a.k_tok, rowbytes, &full_bar[slot]);
       }
+      if (vc) {
+        if (lane == 0) bulk_copy_g2s(vd, a.v + vb + static_cast<int64_t>(rs) * a.v_tok, nr * rowbytes, &full_bar[slot]);
+      } else if (lane < nr) {
+        bulk_copy_g2s(vd + lane * rowbytes, a.v + vb + static_cast<int64_t>(rs + lane) * a.v_tok, rowbytes, &full_bar[slot]);
+      }
+      ++issued;
     }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-      for (int g = 0; g < GM; ++g)
-        if (g < G) {
-#pragma unroll
-          for (int j = 0; j < RB; ++j) sc[g][j] += __shfl_xor_sync(0xffffffffu, sc[g][j], o);
-        }
-    float vr[RB][DPL];
-#pragma unroll
-    for (int j = 0; j < RB; ++j) unpack<DPL>(vraw[j], vr[j]);
+    // the copies still in flight land before the CTA leaves (bounded)
+    if (lane == 0) {
+      const int first = issued > kStages ? issued - kStages : 0;
+      for (int st = first; st < issued; ++st)
+        mbar_wait(&full_bar[st % kStages], (st / kStages) & 1, nullptr, nullptr);
+    }
+    __syncwarp();
+  } else {
+    // --------------------------------------------------------- consumers
+    const int d0 = lane * DPL;
+    float q[GM][DPL];
 #pragma unroll
     for (int g = 0; g < GM; ++g) {
-      if (g >= G) continue;
-      float bm = -INFINITY;
+      const uint16_t* qp = a.q + l * a.q_layer + s * a.q_seq +
+                           static_cast<int64_t>(h * G + (g < G ? g : 0)) * a.q_head + d0;
 #pragma unroll
-      for (int j = 0; j < RB; ++j) {
-        if (!ok[j]) sc[g][j] = -INFINITY;
-        bm = fmaxf(bm, sc[g][j]);
-      }
-      if (bm == -INFINITY) continue;                // (uniform) nothing valid in this batch
-      const float mn = fmaxf(mx[g], bm);
-      const float rescale = fast_exp2(mx[g] - mn);  // 0 on the first valid batch
-      sum[g] *= rescale;
-#pragma unroll
-      for (int i = 0; i < DPL; ++i) acc[g][i] *= rescale;
-#pragma unroll
-      for (int j = 0; j < RB; ++j) {
-        const float p = ok[j] ? fast_exp2(sc[g][j] - mn) : 0.f;
-        sum[g] += p;
-#pragma unroll
-        for (int i = 0; i < DPL; ++i) acc[g][i] = fmaf(p, vr[j][i], acc[g][i]);
-      }
-      mx[g] = mn;
+      for (int i = 0; i < DPL; ++i) q[g][i] = g < G ? bf16f(qp[i]) * a.c1 : 0.f;
     }
-  }
-  // merge the warps' states per head through shared memory
+    const int32_t* idx = nullptr;
+    if (a.keep_idx != nullptr)
+      idx = a.keep_idx + (a.varlen ? (static_cast<int64_t>(l) * a.Hkv + h) * a.Ktot + row0
+                                   : static_cast<int64_t>(u) * a.K_dense);
+    for (int st = 0; st < nst; ++st) {
+      const int slot = st % kStages;
+      const bool got = mbar_wait(&full_bar[slot], (st / kStages) & 1, &abort_flag, a.status);
+      if (!__all_sync(0xffffffffu, got)) break;
+      const int rs = r0 + st * kStageRows;
+      const uint8_t* kst = ks + slot * kStageRows * rowbytes + d0 * 2;
+      const uint8_t* vst = vs + slot * kStageRows * rowbytes + d0 * 2;
 #pragma unroll
-  for (int g = 0; g < GM; ++g) {
-    if (lane == 0) {
-      red[warp][g][0] = mx[g];
-      red[warp][g][1] = sum[g];
+      for (int half = 0; half < kStageRows / kDecWarps / RB; ++half) {
+        const int jr0 = warp * (kStageRows / kDecWarps) + half * RB;   // row within the stage
+        RawDims<DPL> kraw[RB], vraw[RB];
+        bool ok[RB];
+#pragma unroll
+        for (int j = 0; j < RB; ++j) {
+          const int r = rs + jr0 + j;
+          ok[j] = r < r1 && (idx == nullptr || __ldg(idx + (r < r1 ? r : r1 - 1)) >= 0);
+          kraw[j] = *reinterpret_cast<const RawDims<DPL>*>(kst + (jr0 + j) * rowbytes);
+          vraw[j] = *reinterpret_cast<const RawDims<DPL>*>(vst + (jr0 + j) * rowbytes);
+        }
+        float sc[GM][RB];
+#pragma unroll
+        for (int j = 0; j < RB; ++j) {
+          float kr[DPL];
+          unpack<DPL>(kraw[j], kr);
+#pragma unroll
+          for (int g = 0; g < GM; ++g) {
+            float t = 0.f;
+#pragma unroll
+            for (int i = 0; i < DPL; ++i) t = fmaf(q[g][i], kr[i], t);
+            sc[g][j] = t;
+          }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+          for (int g = 0; g < GM; ++g)
+            if (g < G) {
+#pragma unroll
+              for (int j = 0; j < RB; ++j) sc[g][j] += __shfl_xor_sync(0xffffffffu, sc[g][j], o);
+            }
+        // rows past the end hold stale shared memory: their values are
+        // zeroed (a weight of zero would not remove a stale NaN)
+        float vr[RB][DPL];
+#pragma unroll
+        for (int j = 0; j < RB; ++j) {
+          unpack<DPL>(vraw[j], vr[j]);
+#pragma unroll
+          for (int i = 0; i < DPL; ++i) vr[j][i] = ok[j] ? vr[j][i] : 0.f;
+        }
+#pragma unroll
+        for (int g = 0; g < GM; ++g) {
+          if (g >= G) continue;
+          float bm = -INFINITY;
+#pragma unroll
+          for (int j = 0; j < RB; ++j) {
+            if (!ok[j]) sc[g][j] = -INFINITY;
+            bm = fmaxf(bm, sc[g][j]);
+          }
+          if (bm == -INFINITY) continue;            // (uniform) nothing valid here
+          const float mn = fmaxf(mx[g], bm);
+          const float rescale = fast_exp2(mx[g] - mn);
+          sum[g] *= rescale;
+#pragma unroll
+          for (int i = 0; i < DPL; ++i) acc[g][i] *= rescale;
+#pragma unroll
+          for (int j = 0; j < RB; ++j) {
+            const float p = ok[j] ? fast_exp2(sc[g][j] - mn) : 0.f;
+            sum[g] += p;
+#pragma unroll
+            for (int i = 0; i < DPL; ++i) acc[g][i] = fmaf(p, vr[j][i], acc[g][i]);
+          }
+          mx[g] = mn;
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty_bar[slot]);
     }
+    // this warp's state per head, for the merge
 #pragma unroll
-    for (int i = 0; i < DPL; ++i) racc[warp][g][d0 + i] = acc[g][i];
+    for (int g = 0; g < GM; ++g) {
+      if (lane == 0) {
+        red[warp][g][0] = mx[g];
+        red[warp][g][1] = sum[g];
+      }
+#pragma unroll
+      for (int i = 0; i < DPL; ++i) racc[warp][g][d0 + i] = acc[g][i];
+    }
   }
   __syncthreads();
-  for (int g = warp; g < G; g += kDecWarps) {
-    float M = -INFINITY;
+  if (warp < kDecWarps) {
+    const int d0 = lane * DPL;
+    for (int g = warp; g < G; g += kDecWarps) {
+      float M = -INFINITY;
 #pragma unroll
-    for (int w = 0; w < kDecWarps; ++w) M = fmaxf(M, red[w][g][0]);
-    float L = 0.f, o[DPL];
+      for (int w = 0; w < kDecWarps; ++w) M = fmaxf(M, red[w][g][0]);
+      float L = 0.f, o[DPL];
 #pragma unroll
-    for (int i = 0; i < DPL; ++i) o[i] = 0.f;
-    if (M > -INFINITY) {
+      for (int i = 0; i < DPL; ++i) o[i] = 0.f;
+      if (M > -INFINITY) {
 #pragma unroll
-      for (int w = 0; w < kDecWarps; ++w) {
-        const float mw = red[w][g][0];
-        if (mw == -INFINITY) continue;
-        const float f = exp2f(mw - M);
-        L += f * red[w][g][1];
+        for (int w = 0; w < kDecWarps; ++w) {
+          const float mw = red[w][g][0];
+          if (mw == -INFINITY) continue;
+          const float f = exp2f(mw - M);
+          L += f * red[w][g][1];
 #pragma unroll
-        for (int i = 0; i < DPL; ++i) o[i] += f * racc[w][g][d0 + i];
+          for (int i = 0; i < DPL; ++i) o[i] += f * racc[w][g][d0 + i];
+        }
       }
-    }
-    float* out = a.part + ((static_cast<int64_t>(u) * a.n_splits + split) * a.G + g) * (a.d + 2);
+      float* out = a.part + ((static_cast<int64_t>(u) * a.n_splits + split) * a.G + g) * (a.d + 2);
 #pragma unroll
-    for (int i = 0; i < DPL; ++i) out[d0 + i] = o[i];
-    if (lane == 0) {
-      out[a.d] = M;
-      out[a.d + 1] = L;
+      for (int i = 0; i < DPL; ++i) out[d0 + i] = o[i];
+      if (lane == 0) {
+        out[a.d] = M;
+        out[a.d + 1] = L;
+      }
     }
   }
 }
@@ -264,11 +340,18 @@ cudaError_t launch_decode_d(const DecodeArgs& a, cudaStream_t stream) {
   const int64_t grid1 = static_cast<int64_t>(a.n_units) * a.n_splits;
   const int64_t warps2 = static_cast<int64_t>(a.n_units) * a.G;
   const unsigned grid2 = static_cast<unsigned>((warps2 * 32 + 255) / 256);
-  if (a.G <= 4)
-    decode_partial_kernel<DPL, 4><<<static_cast<unsigned>(grid1), kDecWarps * 32, 0, stream>>>(a);
-  else
-    decode_partial_kernel<DPL, 8><<<static_cast<unsigned>(grid1), kDecWarps * 32, 0, stream>>>(a);
-  cudaError_t e = cudaGetLastError();
+  const int smem = decode_smem_bytes(a.d);
+  cudaError_t e;
+  if (a.G <= 4) {
+    e = cudaFuncSetAttribute(decode_partial_kernel<DPL, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    decode_partial_kernel<DPL, 4><<<static_cast<unsigned>(grid1), kDecThreads, smem, stream>>>(a);
+  } else {
+    e = cudaFuncSetAttribute(decode_partial_kernel<DPL, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    decode_partial_kernel<DPL, 8><<<static_cast<unsigned>(grid1), kDecThreads, smem, stream>>>(a);
+  }
+  e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   decode_combine_kernel<DPL><<<grid2, 256, 0, stream>>>(a);
   return cudaGetLastError();

@@ -125,6 +125,7 @@ struct DecodeArgs {
   float* part;                      // [unit][split][G][d + 2]: o (unnormalised), max2, sum
   float* out;                       // fp32 outputs
   int64_t o_layer, o_seq, o_head;
+  int32_t* status;
 };
 
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);

@@ -677,7 +677,8 @@ int rolekv_decode_workspace_size(const rolekv_batch* batch, float budget, size_t
 
 int decode_attention(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k_cache,
                      rolekv_tensor v_cache, const int32_t* keep_idx, float budget, float scale,
-                     float* out, void* workspace, size_t workspace_bytes, void* stream) {
+                     float* out, void* workspace, size_t workspace_bytes, int32_t* status_dev,
+                     void* stream) {
   BatchInfo bi;
   int rc = check_batch(batch, &bi);
   if (rc) return rc;
@@ -739,6 +740,7 @@ int decode_attention(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k
   a.o_seq = static_cast<int64_t>(bi.Hq) * bi.d;
   a.o_layer = a.o_seq * bi.b;
   a.o_head = bi.d;
+  a.status = status_dev;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   stage_begin();
   cudaError_t e = launch_decode(a, st);

@@ -70,7 +70,8 @@ _SIGNATURES = [
      [ctypes.POINTER(BatchDesc), ctypes.c_float, ctypes.POINTER(ctypes.c_size_t)]),
     ("decode_attention", ctypes.c_int,
      [ctypes.POINTER(BatchDesc), Tensor, Tensor, Tensor, ctypes.c_void_p, ctypes.c_float,
-      ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]),
+      ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p,
+      ctypes.c_void_p]),
     ("h2o_score", ctypes.c_int,
      [ctypes.POINTER(BatchDesc), Tensor, Tensor, ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p,
       ctypes.c_size_t, ctypes.c_void_p, ctypes.c_void_p]),
@@ -264,7 +265,7 @@ def cache_desc(t: torch.Tensor, batch: Batch, compacted: bool) -> Tensor:
 def decode_attention(batch: Batch, q: torch.Tensor, k_cache: torch.Tensor, v_cache: torch.Tensor,
                      keep_idx: Optional[torch.Tensor], budget: float, out: torch.Tensor,
                      compacted: bool = True, scale: float = 0.0, ws: Optional[torch.Tensor] = None,
-                     stream=None) -> torch.Tensor:
+                     status: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
     """q bf16 [L][b][Hq][d] -> out fp32 [L][b][Hq][d]."""
     if ws is None:
         ws = decode_workspace(batch, budget, device=q.device)
@@ -274,7 +275,7 @@ def decode_attention(batch: Batch, q: torch.Tensor, k_cache: torch.Tensor, v_cac
     qd = Tensor(q.data_ptr(), sl, ss, sh, q.shape[-1])
     _check(lib().decode_attention(ctypes.byref(batch.desc), qd, cache_desc(k_cache, batch, compacted),
                                   cache_desc(v_cache, batch, compacted), _ptr(keep_idx), budget, scale,
-                                  _ptr(out), _ptr(ws), ws.numel(), _stream(stream)))
+                                  _ptr(out), _ptr(ws), ws.numel(), _ptr(status), _stream(stream)))
     return out
 
 

@@ -222,9 +222,11 @@ def test_decode_attention_compacted(case):
     R.kv_compact(batch, K, V, keep, B, kc, vc)
     qd = I.make_q_decode(w, 7, device=DEV)
     out = torch.full((w.L, w.b, w.Hq, w.d), float("nan"), dtype=torch.float32, device=DEV)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
     for _ in range(2):                               # the workspace holds no state
-        R.decode_attention(batch, qd, kc, vc, keep, B, out)
+        R.decode_attention(batch, qd, kc, vc, keep, B, out, status=status)
     torch.cuda.synchronize()
+    assert int(status.item()) == 0
     ob = oracle_batch(w)
     kb, vb, kp = I.bf16_bits(kc), I.bf16_bits(vc), keep.cpu().numpy()
     cu = ob.kept_offsets(B)
@@ -248,8 +250,35 @@ def test_decode_attention_full_cache(varlen):
     batch = lib_batch(w, DEV)
     qd = I.make_q_decode(w, 8, device=DEV)
     out = torch.empty((w.L, w.b, w.Hq, w.d), dtype=torch.float32, device=DEV)
-    R.decode_attention(batch, qd, K, V, None, 1.0, out, compacted=False)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    R.decode_attention(batch, qd, K, V, None, 1.0, out, compacted=False, status=status)
     torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    ob = oracle_batch(w)
+    kb, vb = I.bf16_bits(K), I.bf16_bits(V)
+    ref = _decode_ref(ob, w, I.bf16_bits(qd), lambda u: ob.kv_rows(kb, u), lambda u: ob.kv_rows(vb, u),
+                      lambda u: np.ones(ob.kv_rows(kb, u).shape[0], dtype=bool))
+    _check_decode(ob, w, out, ref, float(V.float().abs().max()))
+
+
+def test_decode_ignores_stale_stage_rows():
+    """Rows past a unit's last cache row are never read into the result: a
+    decode over a NaN-filled cache first leaves NaN bit patterns in the
+    shared-memory stages, then a cache whose units end in a partial stage
+    must still match the oracle."""
+    w = _w("llama8b", L=2, b=2, Hq=8, Hkv=2, n=1999)
+    roles_np, K, V, _ = _snapkv_inputs(w, seed=9)
+    batch = lib_batch(w, DEV)
+    qd = I.make_q_decode(w, 9, device=DEV)
+    out = torch.empty((w.L, w.b, w.Hq, w.d), dtype=torch.float32, device=DEV)
+    nan_k = torch.full_like(K, float("nan"))
+    for _ in range(3):
+        R.decode_attention(batch, qd, nan_k, nan_k, None, 1.0, out, compacted=False)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    R.decode_attention(batch, qd, K, V, None, 1.0, out, compacted=False, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    assert torch.isfinite(out).all()
     ob = oracle_batch(w)
     kb, vb = I.bf16_bits(K), I.bf16_bits(V)
     ref = _decode_ref(ob, w, I.bf16_bits(qd), lambda u: ob.kv_rows(kb, u), lambda u: ob.kv_rows(vb, u),

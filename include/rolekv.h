@@ -292,6 +292,14 @@ const char* rolekv_last_error(void);
 /* Library version string. */
 const char* rolekv_version(void);
 
+/* Diagnostic (no counterpart in the paper): runs the bounded device wait the
+ * kernels use on a barrier phase that nothing completes, so that it gives up
+ * after limit_ns nanoseconds (0 .. 1e10) and ORs ROLEKV_STATUS_TIMEOUT into
+ * *status_dev (device int32, required); the kernel then returns normally.
+ * It lets a caller check, without a fault, that a stuck wait is reported and
+ * the context stays usable. */
+int rolekv_selftest_wait(int64_t limit_ns, int32_t* status_dev, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

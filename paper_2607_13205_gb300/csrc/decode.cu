@@ -333,7 +333,25 @@ __global__ void __launch_bounds__(256) decode_combine_kernel(const DecodeArgs a)
   for (int i = 0; i < DPL; ++i) dst[i] = L > 0.f ? o[i] / L : 0.f;
 }
 
+// Diagnostic: the bounded mbarrier wait of the kernels above, on a phase that
+// nothing completes, so that it runs out after limit_ns and records
+// ROLEKV_STATUS_TIMEOUT; the CTA then returns normally.
+__global__ void selftest_wait_kernel(uint64_t limit_ns, int32_t* status) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  mbar_wait_for(&bar, 0, nullptr, status, limit_ns);   // phase 0 never completes
+}
+
 }  // namespace
+
+cudaError_t launch_selftest_wait(uint64_t limit_ns, int32_t* status, cudaStream_t stream) {
+  selftest_wait_kernel<<<1, 32, 0, stream>>>(limit_ns, status);
+  return cudaGetLastError();
+}
 
 template <int DPL>
 cudaError_t launch_decode_d(const DecodeArgs& a, cudaStream_t stream) {

@@ -61,23 +61,28 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Bounded wait for the phase of `bar` with the given parity.  Returns false if
-// the CTA-wide abort flag (may be null) is raised or the time limit passes;
-// on a timeout the flag is raised and ROLEKV_STATUS_TIMEOUT recorded.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                          int32_t* status) {
+// the CTA-wide abort flag (may be null) is raised or `limit_ns` passes; on a
+// timeout the flag is raised and ROLEKV_STATUS_TIMEOUT recorded.
+__device__ __forceinline__ bool mbar_wait_for(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                              int32_t* status, uint64_t limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((it & 15u) == 0) {
       if (abort_flag != nullptr && *abort_flag) return false;
-      if (global_timer_ns() - t0 > kWaitLimitNs) {
+      if (global_timer_ns() - t0 > limit_ns) {
         if (abort_flag != nullptr) *abort_flag = 1;
         if (status != nullptr) atomicOr(status, ROLEKV_STATUS_TIMEOUT);
         return false;
       }
     }
   }
+}
+
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                          int32_t* status) {
+  return mbar_wait_for(bar, parity, abort_flag, status, kWaitLimitNs);
 }
 
 // --------------------------------------------------------------------- TMA --

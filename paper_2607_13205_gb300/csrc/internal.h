@@ -129,6 +129,7 @@ struct DecodeArgs {
 };
 
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
+cudaError_t launch_selftest_wait(uint64_t limit_ns, int32_t* status, cudaStream_t stream);
 
 // Compaction -----------------------------------------------------------------
 

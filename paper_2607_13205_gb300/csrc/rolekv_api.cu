@@ -471,6 +471,16 @@ const char* rolekv_last_error(void) { return g_err; }
 
 const char* rolekv_version(void) { return "rolekv 0.1 (sm_103a)"; }
 
+int rolekv_selftest_wait(int64_t limit_ns, int32_t* status_dev, void* stream) {
+  if (status_dev == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "status_dev is NULL");
+  if (limit_ns < 0 || limit_ns > 10000000000LL)
+    return fail(ROLEKV_ERR_INVALID_ARG, "limit_ns=%lld outside 0..1e10", static_cast<long long>(limit_ns));
+  cudaError_t e = launch_selftest_wait(static_cast<uint64_t>(limit_ns), status_dev,
+                                       static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "rolekv_selftest_wait");
+  return ROLEKV_OK;
+}
+
 int rolekv_workspace_size(int op, const rolekv_batch* batch, int32_t W, size_t* bytes) {
   if (bytes == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "bytes is NULL");
   BatchInfo bi;

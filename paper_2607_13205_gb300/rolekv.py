@@ -66,6 +66,7 @@ _SIGNATURES = [
     ("quest_score", ctypes.c_int,
      [ctypes.POINTER(BatchDesc), Tensor, Tensor, ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p,
       ctypes.c_void_p]),
+    ("rolekv_selftest_wait", ctypes.c_int, [ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]),
     ("rolekv_decode_workspace_size", ctypes.c_int,
      [ctypes.POINTER(BatchDesc), ctypes.c_float, ctypes.POINTER(ctypes.c_size_t)]),
     ("decode_attention", ctypes.c_int,
@@ -245,6 +246,10 @@ def quest_score(batch: Batch, q_win: torch.Tensor, k: torch.Tensor, W: int, page
     _check(lib().quest_score(ctypes.byref(batch.desc), tensor_desc(q_win, False),
                              tensor_desc(k, batch.varlen), W, page, _ptr(scores), _stream(stream)))
     return scores
+
+
+def selftest_wait(limit_ns: int, status: torch.Tensor, stream=None) -> None:
+    _check(lib().rolekv_selftest_wait(int(limit_ns), _ptr(status), _stream(stream)))
 
 
 def decode_workspace(batch: Batch, budget: float, device="cuda") -> torch.Tensor:

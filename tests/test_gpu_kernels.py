@@ -539,3 +539,19 @@ def test_rolekv_compress_pipeline(name):
             kr = ko.reshape(ob.n_units, -1, w.d)[u]
         check_index_sets(ob, u, row, pooled, roles_np, I.N_ROLES, I.PAPER_ALPHA, I.ROLE_KEY, 0.0, B)
         assert np.array_equal(kr, O.compact_unit(ob.kv_rows(kb, u), row))
+
+
+def test_bounded_wait_reports_timeout():
+    """A device wait that nothing satisfies gives up after its limit, records
+    STATUS_TIMEOUT, and leaves the context usable for the next launch."""
+    import time
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    R.selftest_wait(20_000_000, status)          # 20 ms
+    torch.cuda.synchronize()
+    dt = time.perf_counter() - t0
+    assert int(status.item()) & R.STATUS_TIMEOUT
+    assert 0.015 <= dt < 5.0
+    x = torch.arange(8, device=DEV).sum()        # the context still works
+    assert int(x.item()) == 28

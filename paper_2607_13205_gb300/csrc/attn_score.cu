@@ -922,7 +922,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         ++qload;
         // the chunk's key tiles, once for each pass
         bool ok = true;
-        for (int pass = 0; pass < 2 && ok; ++pass)
+        for (int pass = fa.single; pass < 2 && ok; ++pass)
           for (int kt = kt0; kt < kt1; ++kt) {
             const int slot = kload % C::SK;
             if (!mbar_wait(&sh.k_empty[slot], ((kload / C::SK) & 1) ^ 1, sh.abort_flag, a.status)) {
@@ -962,7 +962,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait(sh.q_full, quse & 1, sh.abort_flag, a.status)) break;
         ++quse;
         const uint32_t qbase = smem_u32(sh.q);
-        for (int pass = 0; pass < 2 && ok; ++pass)
+        for (int pass = fa.single; pass < 2 && ok; ++pass)
           for (int kt = kt0; kt < kt1; ++kt) {
             const int kslot = kuse % C::SK;
             const int ab = pair & 1;
@@ -1026,6 +1026,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int kt0, kt1;
       chunk_tiles(a, n, chunk, &kt0, &kt1);
 
+      if (!fa.single) {
       // ---- pass 1: running (max2, sum) of this thread's row over its keys
       const int pos = row_position(a, n, 0, row);
       float m2 = -INFINITY, l = 0.f;
@@ -1090,12 +1091,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       ok = __all_sync(0xffffffffu, mbar_wait(sh.lse_go, ipop & 1, sh.abort_flag, a.status));
       if (!ok || *sh.abort_flag) break;
-      // ---- normalisers of the unit's rows from all chunks' partials
+      }  // pass 1
+      // ---- normalisers of the unit's rows from all chunks' partials (or,
+      // with caller-supplied window normalisers, as snapkv_lse_kernel wrote them)
       if (etid < kRowsMax) {
         const int j = etid;
         const int p = row_position(a, n, 0, j);
         float nl = -INFINITY;
-        if (p >= 0) {
+        if (fa.single) {
+          nl = (p >= 0) ? a.lse2[static_cast<int64_t>(u) * kRowsMax + j] : -INFINITY;
+        } else if (p >= 0) {
           // one online merge over the chunks, eight independent loads in flight
           const float2* part_j = a.partials + static_cast<int64_t>(u) * a.n_chunks * kRowsMax + j;
           float m = -INFINITY, s = 0.f;

@@ -48,6 +48,7 @@ struct FusedArgs {
   ScoreArgs s;                      // s.n_chunks = chunks per unit, s.chunk_tiles = tiles per chunk
   int32_t* work;                    // [1 + u]: chunks of unit u done with pass 1 ([0] unused)
   int32_t n_items;
+  int32_t single;                   // 1: normalisers given in s.lse2, pass 2 only
 };
 
 cudaError_t launch_snapkv_fused(int d, const CUtensorMap& kmap, const CUtensorMap& qmap,

@@ -296,14 +296,21 @@ int run_snapkv(const BatchInfo& bi, const int32_t* cu_seqlens, const rolekv_tens
   rc = make_row_map(&qmap, q_win, tensor_span(q_win, bi.L, bi.b, bi.Hq, W, bi.d, false), W);
   if (rc) return rc;
   cudaError_t e;
-  if (lse_win == nullptr && p.fused) {
-    // one persistent launch: both passes, normalisers formed in-kernel
+  if (p.fused) {
+    // one persistent launch: both passes with the normalisers formed
+    // in-kernel, or pass 2 alone after the caller's normalisers are converted
     FusedArgs fa;
     fa.s = a;
     fa.work = p.work;
     fa.n_items = p.n_items;
-    e = cudaMemsetAsync(p.work, 0, (static_cast<size_t>(a.n_units) + 1) * 4, stream);
-    if (e != cudaSuccess) return cuda_fail(e, "clearing the work counters");
+    fa.single = lse_win != nullptr;
+    if (fa.single) {
+      e = launch_snapkv_lse(a, lse_win, stream);
+      if (e != cudaSuccess) return cuda_fail(e, "snapkv normalisers");
+    } else {
+      e = cudaMemsetAsync(p.work, 0, (static_cast<size_t>(a.n_units) + 1) * 4, stream);
+      if (e != cudaSuccess) return cuda_fail(e, "clearing the work counters");
+    }
     e = launch_snapkv_fused(bi.d, kmap, qmap, fa, stream);
     if (e != cudaSuccess) return cuda_fail(e, "snapkv fused score");
     stage_mark(stream);

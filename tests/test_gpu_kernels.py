@@ -59,9 +59,10 @@ def test_snapkv_score_matches_oracle(case):
             assert abs(ob.score_view(gpre, u).astype(np.float64).sum() - min(w.W, n) * w.G) < 1e-3 * min(w.W, n) * w.G
 
 
-def test_snapkv_with_supplied_lse():
+@pytest.mark.parametrize("case", ["varlen_short_empty", "two_row_tiles_w64_multichunk"])
+def test_snapkv_with_supplied_lse(case):
     """Single pass with the window rows' normalisers given (natural log)."""
-    w = SNAPKV_CASES["varlen_short_empty"]
+    w = SNAPKV_CASES[case]
     roles, K, V, qw = _snapkv_inputs(w, seed=3)
     ob = oracle_batch(w)
     kb, qb = I.bf16_bits(K), I.bf16_bits(qw)

@@ -50,8 +50,9 @@ struct Cfg {
   static constexpr int kQSlotBytes = kRowsMax * D * 2;   // one 256-row query block
   static constexpr int kKHalfBytes = kTileKeys * 128;
   static constexpr int kQHalfBytes = kRowsMax * 128;
-  static constexpr int SQ = (PASS == kPassColsum) ? 2 : 1;
-  static constexpr int SK = (PASS == kPassColsum) ? 2 : 4;
+  // every CTA keeps one query block and streams key tiles
+  static constexpr int SQ = 1;
+  static constexpr int SK = 4;
   static constexpr int kQOff = 0;
   static constexpr int kKOff = kQOff + SQ * kQSlotBytes;
   static constexpr int kLseOff = kKOff + SK * kKTileBytes;
@@ -215,18 +216,15 @@ __device__ __forceinline__ Work decode_work(const ScoreArgs& a, int pass) {
     w.kt1 = min(ntiles, w.kt0 + a.chunk_tiles);
     w.rb0 = 0;
     w.rb1 = n > 0 ? 1 : 0;
-  } else if (pass == kPassRowstats) {
+  } else {
+    // H2O, both passes: one query block, the key tiles up to its last
+    // position (pass 2 adds its column sums into the scores atomically)
     const int rb = a.nrb_max - 1 - slot;        // longest query blocks first
     w.rb0 = rb;
     w.rb1 = (rb * a.P < n) ? rb + 1 : rb;
     const int kend = min(n, (rb + 1) * a.P);
     w.kt0 = 0;
     w.kt1 = (kend + kTileKeys - 1) / kTileKeys;
-  } else {
-    w.kt0 = slot;
-    w.kt1 = (slot < ntiles) ? slot + 1 : slot;
-    w.rb0 = (slot * kTileKeys) / a.P;
-    w.rb1 = num_row_blocks(a, n);
   }
   if (w.kt1 <= w.kt0 || w.rb1 <= w.rb0) {
     w.kt1 = w.kt0;
@@ -489,7 +487,12 @@ __device__ __forceinline__ void colsum_epilogue(const ScoreArgs& a, const Work& 
 #pragma unroll
       for (int x = 1; x < kParts; ++x) total += sh.red[(x - 1) * kTileKeys + kl];
       mbar_arrive(sh.red_empty);
-      if (t < n) a.prepool[sbase + t] = total;
+      if (t < n) {
+        if (a.mode == kModeH2O)
+          atomicAdd(a.prepool + sbase + t, total);   // one query block's share
+        else
+          a.prepool[sbase + t] = total;
+      }
     }
     ++xchg;
   }
@@ -510,9 +513,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const Work w = decode_work(a, PASS);
   const int nrt = a.nrows_pad / 128;
   const int n = w.unit.n;
-  // Pass 2 of H2O streams query blocks against one key tile; every other
-  // combination keeps one query block for the whole CTA.
-  const bool q_streams = (PASS == kPassColsum) && (a.mode == kModeH2O);
+  // Every CTA keeps one query block for its whole life and streams key tiles.
+  const bool q_streams = false;
 
   // ---- set-up: barriers, zeroed padding rows, tensor memory
   if (threadIdx.x == 0) {

@@ -239,7 +239,7 @@ int plan_score(int mode, const BatchInfo& bi, int W, bool need_partials, bool ne
   } else {
     a.nrb_max = (bi.n_max + a.P - 1) / a.P;
     p->grid1 = a.n_units * a.nrb_max;
-    p->grid2 = a.n_units * ntiles;
+    p->grid2 = p->grid1;                          // pass 2 per query block too
   }
   size_t off = 256;   // first 256 bytes reserved
   p->off_partials = off;
@@ -568,6 +568,9 @@ int h2o_score(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k, float
   stage_begin();
   cudaError_t e = launch_attn_pass(0, bi.d, kmap, qmap, a, p.grid1, st);
   if (e != cudaSuccess) return cuda_fail(e, "h2o pass 1");
+  // pass 2 adds every query block's column sums into the scores
+  e = cudaMemsetAsync(scores, 0, static_cast<size_t>(score_elems(bi)) * sizeof(float), st);
+  if (e != cudaSuccess) return cuda_fail(e, "clearing the scores");
   stage_mark(st);
   e = launch_attn_pass(1, bi.d, kmap, qmap, a, p.grid2, st);
   if (e != cudaSuccess) return cuda_fail(e, "h2o pass 2");

@@ -219,6 +219,8 @@ def run_gpu(args):
     stream = torch.cuda.current_stream(dev)
 
     names = ["pass1", "pass2", "select", "compact"] if h2o else ["score", "select", "compact"]
+    # the Quest page bound is selected as it is (no max-pool over the KV axis)
+    pool_k = 1 if args.score == "quest" else w.pool_k
     ns = len(names) - 2                              # score kernels
 
     def score():
@@ -238,7 +240,7 @@ def run_gpu(args):
         score()
         if ev is not None:
             R.set_stage_events(ev[1 + ns:2 + ns])
-        R.role_alloc_select(batch, scores, roles, params, keep, pool_k=w.pool_k, status=status,
+        R.role_alloc_select(batch, scores, roles, params, keep, pool_k=pool_k, status=status,
                             stream=stream)
         if ev is not None:
             R.set_stage_events(ev[2 + ns:3 + ns])
@@ -500,7 +502,7 @@ def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_o
         V.copy_(h_v, non_blocking=True)
         roles.copy_(h_roles, non_blocking=True)
         score()
-        R.role_alloc_select(batch, scores, roles, params, keep, pool_k=w.pool_k, status=status,
+        R.role_alloc_select(batch, scores, roles, params, keep, pool_k=(1 if args.score == "quest" else w.pool_k), status=status,
                             stream=stream)
         R.kv_compact(batch, K, V, keep, B, k_out, v_out, status=status, stream=stream)
         o_keep.copy_(keep, non_blocking=True)

@@ -15,16 +15,20 @@
 //   pass 1  load, pool, key; per role, a histogram of the key's bits
 //           30..31-NB (the top bit is shared by every key when all scores
 //           have one sign): exponent and leading mantissa bits.  The role
-//           counts are the histograms' sums.
+//           counts are the histograms' sums.  Under GLOBAL there is one
+//           bucket, so one histogram of every eligible token.
 //   quotas  one warp, lane r for role r (water-filling, largest remainders).
-//   first digit from the pass-1 histograms, per bucket.
-//   pass 2  every token is decided (kept / dropped) unless its first digit is
-//           its bucket's threshold digit; those "candidates" (a few percent)
-//           go to a list in shared memory.
+//   first digit from the pass-1 histograms, per bucket; while the keys at
+//           the threshold digits would overflow the list, a full pass over
+//           the slots per 8 more bits.
+//   pass 2  every token is decided (kept / dropped) unless its key prefix is
+//           its bucket's threshold prefix; those "candidates" (a few
+//           percent) go to a list in shared memory.
 //   list    the remaining bits in 8-bit rounds over the list; ties at the
 //           threshold are ranked in index order; the kept ones join the bits.
 // A unit with a NaN, keys of both signs, or more candidates than the list
-// holds takes the general path: four 8-bit rounds over all slots.
+// holds 4 to 5 bits above the bottom takes the general path: four 8-bit
+// rounds over all slots.
 // Kept positions are then written in ascending order from a block-wide scan
 // of the bit words.
 #include <cuda_runtime.h>
@@ -161,10 +165,10 @@ __device__ __forceinline__ uint32_t floor_bits(int s0, int nf, int n) {
 }
 
 // Pass 1 for a pool half-width HW known at compile time.
-template <int HW, int NT>
-__device__ __forceinline__ void pass1(const UnitView& v, int n_roles, int nb, uint4* keys4,
-                                      uint32_t* hist16, int32_t* floor_role, bool& nan_hint,
-                                      uint32_t& top_and, uint32_t& top_or) {
+template <int HW, int NT, bool GL>
+__device__ __forceinline__ void pass1(const UnitView& v, int n_roles, uint32_t ban, int nb,
+                                      uint4* keys4, uint32_t* hist16, int32_t* floor_role,
+                                      bool& nan_hint, uint32_t& top_and, uint32_t& top_or) {
   constexpr int NB = (HW + 3) / 4;   // neighbour groups on each side
   const int sh0 = 31 - nb;
   const uint32_t bmask = (1u << nb) - 1u;
@@ -207,7 +211,8 @@ __device__ __forceinline__ void pass1(const UnitView& v, int n_roles, int nb, ui
         top_and &= k[j];
         top_or |= k[j];
         const uint32_t bin = (k[j] >> sh0) & bmask;
-        atomicAdd(&hist16[r * words_per_role + (bin >> 1)], 1u << (16 * (bin & 1u)));
+        if (!GL || !((ban >> r) & 1u))
+          atomicAdd(&hist16[(GL ? 0u : r) * words_per_role + (bin >> 1)], 1u << (16 * (bin & 1u)));
       }
     }
   }
@@ -235,7 +240,7 @@ __device__ void quotas_warp(const SelectArgs& a, int lane, int64_t K_full, SelSh
                                                          : a.alpha_fx[r];
   int64_t q = 0, bsize = 0;
   if (a.policy == ROLEKV_POLICY_GLOBAL) {
-    const int64_t elig = sum8((valid && !banned) ? cnt : 0);
+    const int64_t elig = S.count[0];   // every eligible token, counted in row 0
     if (r == 0) {
       q = K_full < elig ? K_full : elig;
       bsize = elig;
@@ -336,6 +341,7 @@ __device__ void descend(SelShared& S, int b, int lane, int shift) {
     const int need2 = need - gb;
     S.prefix[b] = prefix;
     S.need[b] = need2;
+    S.cand[b] = ad;
     if (shift == 0) {
       // ad keys of the bucket equal the threshold; need2 of them are kept
       S.thr[b] = (need2 >= ad) ? prefix : prefix + 1u;
@@ -355,31 +361,14 @@ __device__ void descend_first(const SelectArgs& a, SelShared& S, const uint32_t*
   constexpr int nb = NB;
   constexpr int wpl = 1 << (nb - 6);   // histogram words (two bins each) per lane
   constexpr int wpr = 1 << (nb - 1);   // words per role
-  const uint32_t roles = (a.policy == ROLEKV_POLICY_GLOBAL)
-                             ? (((1u << a.n_roles) - 1u) & ~a.ban_mask)
-                             : (1u << b);
-  // counts of bins 2w (low half) and 2w+1 (high half), summed over the roles;
-  // a bin holds at most n < 65536 tokens, so the halves never carry
-  const bool single = (roles & (roles - 1)) == 0;
-  const uint32_t* h0 = hist16 + (__ffs(roles) - 1) * wpr;
-  auto word = [&](int w) {
-    if (single) return h0[w];
-    uint32_t x = 0;
-    for (uint32_t m = roles; m != 0; m &= m - 1) x += hist16[(__ffs(m) - 1) * wpr + w];
-    return x;
-  };
+  // counts of bins 2w (low half) and 2w+1 (high half); a bin holds at most
+  // n < 65536 tokens, so the halves never carry
+  const uint32_t* h0 = hist16 + b * wpr;
   int mine = 0;
-  if (single) {
 #pragma unroll
-    for (int i = 0; i < wpl; ++i) {
-      const uint32_t x = h0[lane * wpl + ((i + lane) & (wpl - 1))];
-      mine += static_cast<int>((x & 0xFFFFu) + (x >> 16));
-    }
-  } else {
-    for (int i = 0; i < wpl; ++i) {
-      const uint32_t x = word(lane * wpl + ((i + lane) & (wpl - 1)));
-      mine += static_cast<int>((x & 0xFFFFu) + (x >> 16));
-    }
+  for (int i = 0; i < wpl; ++i) {
+    const uint32_t x = h0[lane * wpl + ((i + lane) & (wpl - 1))];
+    mine += static_cast<int>((x & 0xFFFFu) + (x >> 16));
   }
   int incl = mine;   // tokens in this lane's bins or above
 #pragma unroll
@@ -397,7 +386,7 @@ __device__ void descend_first(const SelectArgs& a, SelShared& S, const uint32_t*
   const int F = __ffs(who) - 1;
   const int aboveF = __shfl_sync(0xffffffffu, above, F);
   const int needF = need - aboveF;
-  const uint32_t x = lane < wpl ? word(F * wpl + lane) : 0u;
+  const uint32_t x = lane < wpl ? h0[F * wpl + lane] : 0u;
   const int lo = static_cast<int>(x & 0xFFFFu), hi = static_cast<int>(x >> 16);
   const int pair = lo + hi;
   int incl2 = pair;
@@ -528,6 +517,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
   uint32_t* hist16 = region;                    // pass 1 histograms
   uint32_t* list = region;                      // then the candidate list
   const int list_cap = static_cast<int>(region_bytes(a.n_max) / 4);
+  const bool global = a.policy == ROLEKV_POLICY_GLOBAL;
 
   if (tid < kR) {
     S.count[tid] = 0;
@@ -572,16 +562,24 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
   {
     bool nan_hint = false;
     uint32_t tand = 0xFFFFFFFFu, tor = 0u;
+    // GLOBAL: one histogram (row 0) of every eligible token; otherwise one
+    // row per role
+#define ROLEKV_PASS1(HWV)                                                                   \
+  (global ? pass1<HWV, NT, true>(v, a.n_roles, a.ban_mask, nb, keys4, hist16, S.floor_role, \
+                                 nan_hint, tand, tor)                                       \
+          : pass1<HWV, NT, false>(v, a.n_roles, a.ban_mask, nb, keys4, hist16, S.floor_role, \
+                                  nan_hint, tand, tor))
     switch (a.pool_k >> 1) {
-      case 0: pass1<0, NT>(v, a.n_roles, nb, keys4, hist16, S.floor_role, nan_hint, tand, tor); break;
-      case 1: pass1<1, NT>(v, a.n_roles, nb, keys4, hist16, S.floor_role, nan_hint, tand, tor); break;
-      case 2: pass1<2, NT>(v, a.n_roles, nb, keys4, hist16, S.floor_role, nan_hint, tand, tor); break;
-      case 3: pass1<3, NT>(v, a.n_roles, nb, keys4, hist16, S.floor_role, nan_hint, tand, tor); break;
-      case 4: pass1<4, NT>(v, a.n_roles, nb, keys4, hist16, S.floor_role, nan_hint, tand, tor); break;
-      case 5: pass1<5, NT>(v, a.n_roles, nb, keys4, hist16, S.floor_role, nan_hint, tand, tor); break;
-      case 6: pass1<6, NT>(v, a.n_roles, nb, keys4, hist16, S.floor_role, nan_hint, tand, tor); break;
-      default: pass1<7, NT>(v, a.n_roles, nb, keys4, hist16, S.floor_role, nan_hint, tand, tor); break;
+      case 0: ROLEKV_PASS1(0); break;
+      case 1: ROLEKV_PASS1(1); break;
+      case 2: ROLEKV_PASS1(2); break;
+      case 3: ROLEKV_PASS1(3); break;
+      case 4: ROLEKV_PASS1(4); break;
+      case 5: ROLEKV_PASS1(5); break;
+      case 6: ROLEKV_PASS1(6); break;
+      default: ROLEKV_PASS1(7); break;
     }
+#undef ROLEKV_PASS1
     tand = __reduce_and_sync(0xffffffffu, tand);
     tor = __reduce_or_sync(0xffffffffu, tor);
     const bool nh = __any_sync(0xffffffffu, nan_hint);
@@ -594,10 +592,10 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
   __syncthreads();
 
   // Role counts: the sums of the roles' histograms (a warp's 32 words belong
-  // to one role).
+  // to one role); GLOBAL: the eligible total, in count[0].
   {
     const int wpr = 1 << (nb - 1);
-    for (int x0 = warp * 32; x0 < a.n_roles * wpr; x0 += NT) {
+    for (int x0 = warp * 32; x0 < (global ? 1 : a.n_roles) * wpr; x0 += NT) {
       const uint32_t w = hist16[x0 + lane];
       const int c = warp_sum(static_cast<int>((w & 0xFFFFu) + (w >> 16)));
       if (lane == 0 && c) atomicAdd(&S.count[x0 >> (nb - 1)], c);
@@ -650,20 +648,47 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
         descend_first<10>(a, S, hist16, warp, lane);
     }
     __syncthreads();
-    if (tid == 0) {
-      int total = 0;
-      for (int b = 0; b < kR; ++b) total += S.mode[b] == 2 ? S.cand[b] : 0;
-      if (total > list_cap) S.general = 1;
+  }
+  // While the keys at the buckets' first digits overflow the list (scores in
+  // a narrow range, such as page bounds), one full pass per 8 more bits.
+  int shd = 31 - nb;   // key bits below the decided prefixes
+  if (any_thr && !S.general) {
+    auto cand_total = [&]() {
+      int t = 0;
+      for (int b = 0; b < kR; ++b) t += S.mode[b] == 2 ? S.cand[b] : 0;
+      return t;
+    };
+    while (cand_total() > list_cap && shd > 8) {
+      const int shift = shd - 8;
+      for (int i = 0; i < iters; ++i) {
+        const int g = i * NT + tid;
+        if (g >= ngroups) break;
+        const uint4 kv = keys4[g];
+        const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
+        const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
+        const uint32_t fb = floor_bits(4 * g - off, v.nf, n);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t c = static_cast<uint32_t>(S.code_of_role[(rw >> (8 * j)) & 0xFFu]);
+          if (c >= static_cast<uint32_t>(kR) || ((fb >> j) & 1u)) continue;
+          if ((kk[j] >> shd) != (S.prefix[c] >> shd)) continue;
+          atomicAdd(&S.hist[c][(kk[j] >> shift) & 0xFFu], 1);
+        }
+      }
+      __syncthreads();
+      if (warp < kR && S.mode[warp] == 2) descend(S, warp, lane, shift);
+      __syncthreads();
+      shd = shift;
     }
+    if (tid == 0 && cand_total() > list_cap) S.general = 1;
     __syncthreads();
   }
 
-  const int sh0 = 31 - nb;
   if (!S.general) {
     for (int x = tid; x < 256; x += NT) {
       const uint32_t code = static_cast<uint32_t>(S.code_of_role[x]);
       S.first_of_role[x] = code == kCodeKeep                  ? -1
-                           : code < static_cast<uint32_t>(kR) ? static_cast<int32_t>(S.prefix[code] >> sh0)
+                           : code < static_cast<uint32_t>(kR) ? static_cast<int32_t>(S.prefix[code] >> shd)
                                                                : 0x7FFFFFFF;
     }
     __syncthreads();
@@ -690,7 +715,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
         for (int j = 0; j < 4; ++j) {
           const uint32_t r = (rw >> (8 * j)) & 0xFFu;
           const int T = S.first_of_role[r];
-          const int hb = static_cast<int>(kk[j] >> sh0);
+          const int hb = static_cast<int>(kk[j] >> shd);
           m4 |= static_cast<uint32_t>(hb > T) << j;
           if (hb == T && !((fb >> j) & 1u)) {
             c4 |= 1u << j;
@@ -731,7 +756,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
     if (any_thr) {
       // ---- remaining bits over the candidate list
       const int m = S.list_n;
-      for (int lo = sh0; lo > 0;) {
+      for (int lo = shd; lo > 0;) {
         const int d = lo < 8 ? lo : 8;
         const int shift = lo - d;
         for (int e = tid; e < m; e += NT) {

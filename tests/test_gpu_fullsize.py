@@ -230,4 +230,10 @@ def test_quest_long_full_size():
         assert np.all(np.abs(sc[u] - ref) <= tol)
         check_index_sets(v.ob, 0, kp[u], ref, v.roles, I.N_ROLES, I.PAPER_ALPHA, I.ROLE_KEY, 0.0, B,
                          policy=O.POLICY_GLOBAL)
+        # on the kernel's own page bounds the selection is bit-exact (these
+        # narrow-range, page-constant keys take the selector's extra digit
+        # rounds and its tie ranking)
+        exact = O.select_batch(ob, {u: sc[u].astype(np.float64)}, roles_np, I.N_ROLES, I.PAPER_ALPHA,
+                               I.ROLE_KEY, 0.0, B, O.POLICY_GLOBAL)
+        assert np.array_equal(kp[u], exact[u][0])
         assert np.array_equal(ko[u], O.compact_unit(v.k[0, 0, 0], kp[u]))

@@ -364,6 +364,50 @@ def test_role_alloc_select_bit_exact(case):
             assert per[I.ROLE_KEY] == 0
 
 
+NARROW_CASES = [
+    # (name, n, policy, pool_k, spread): page-constant scores in [2, 2 + spread)
+    ("narrow_quota", 20000, 0, 1, 0.2),
+    ("narrow_global_pool7", 20000, 1, 7, 0.2),
+    ("narrow_fair_short", 9000, 2, 1, 0.2),
+    ("constant_global", 20000, 1, 1, 0.0),
+    ("constant_quota_pool5", 12000, 0, 5, 0.0),
+]
+
+
+@pytest.mark.parametrize("case", NARROW_CASES, ids=[c[0] for c in NARROW_CASES])
+def test_select_narrow_page_constant_scores(case):
+    """Scores constant over pages of 16 and packed into a narrow range (as
+    Quest page bounds are): most keys share the first digit, so the selector
+    takes extra digit rounds before listing candidates; a constant row leaves
+    only ties.  Bit-exact against the oracle on the same scores."""
+    name, n, policy, pool_k, spread = case
+    w = _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=n)
+    roles_np = I.workload_roles(w, 3)
+    batch = lib_batch(w, DEV)
+    g = torch.Generator().manual_seed(17)
+    npages = (n + 15) // 16
+    pages = 2.0 + spread * torch.rand((batch.n_units, npages), generator=g)
+    sc = pages.repeat_interleave(16, dim=1)[:, :n].reshape(batch.score_shape()).contiguous()
+    scores = sc.to(DEV)
+    B = 0.10
+    params = R.select_params(B, I.PAPER_ALPHA, alpha_key=0.0, key_role=I.ROLE_KEY, policy=policy)
+    keep = torch.full(batch.kept_shape(B), -7, dtype=torch.int32, device=DEV)
+    per_role = torch.full((batch.n_units, I.N_ROLES), -1, dtype=torch.int32, device=DEV)
+    R.role_alloc_select(batch, scores, torch.as_tensor(roles_np, device=DEV), params, keep,
+                        pool_k=pool_k, kept_per_role=per_role)
+    torch.cuda.synchronize()
+    ob = oracle_batch(w)
+    scn = sc.numpy()
+    unit_scores = {u: O.maxpool1d(ob.score_view(scn, u).astype(np.float64), pool_k)
+                   for u in range(ob.n_units)}
+    ref = O.select_batch(ob, unit_scores, roles_np, I.N_ROLES, I.PAPER_ALPHA, I.ROLE_KEY, 0.0, B,
+                         policy)
+    got, pr = keep.cpu().numpy().reshape(ob.n_units, -1), per_role.cpu().numpy()
+    for u, (idx, per) in ref.items():
+        assert np.array_equal(got[u], idx), f"{name} unit {u}"
+        assert list(pr[u]) == per, f"{name} unit {u} per-role counts"
+
+
 @pytest.mark.parametrize("akey", [0.0, 0.02])
 def test_select_six_role_taxonomy(akey):
     """The paper's six labels (KEY, VALUE, DELIM, HEADER, PROSE, WS) with its

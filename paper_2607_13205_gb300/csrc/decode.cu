@@ -4,14 +4,17 @@
 //   o_g = sum_j softmax_j(scale q_g . k_j) v_j
 // over the unit's cache rows (the kept slots; -1 slots of an infeasible budget
 // are skipped; with budget 1 and no index the full cache).  Memory-bound: the
-// cache rows are read once.  Split-K: CTA (unit, split) takes 512 rows.  A
-// producer warp streams them into four shared-memory stages of 32 K rows and
-// 32 V rows with bulk copies (one per stage when a unit's rows are
-// contiguous, one per row otherwise), so the bytes in flight do not depend on
-// registers; each of four consumer warps takes 8 rows of every stage for all
-// G query heads, lanes over the head dimension: the G x rows dot products are
-// reduced across the warp and an online softmax per head keeps (max, sum,
-// unnormalised output) in log2 units.  Every wait is a bounded mbarrier wait.
+// cache rows are read once.  Split-K: CTA (unit, split) takes up to 1024 rows
+// (a unit's splits equal in length).  A producer warp streams them into two
+// shared-memory stages of 64 K rows and 64 V rows with bulk copies (K one
+// copy per row, into rows padded by 16 bytes; V one copy per stage when the
+// rows are contiguous).  Each of four consumer warps takes 16 rows of a stage:
+// the G x 16 dot products are one m16n8k16 bf16 MMA tile per 16 dimensions
+// (cache rows x query heads padded to 8, fp32 accumulate), so no cross-lane
+// reduction is needed; the online softmax (log2 units) runs in that fragment
+// layout, and the probabilities and rescale factors pass through a per-warp
+// shared buffer to the output accumulation, where the lanes run over the head
+// dimension with packed f32x2 FMAs.  Every wait is a bounded mbarrier wait.
 // The warps merge through shared memory; a second launch merges the splits of
 // each (unit, head).
 #include <cuda_runtime.h>
@@ -25,28 +28,11 @@
 namespace rolekv {
 namespace {
 
-constexpr int kRowBatch = 8;
-
-__device__ __forceinline__ float bf16f(uint16_t x) { return __uint_as_float(static_cast<uint32_t>(x) << 16); }
-
 // DPL consecutive bf16 values: raw bits, then fp32.
 template <int DPL>
 struct RawDims {
   uint32_t w[DPL / 2];
 };
-
-template <int DPL>
-__device__ __forceinline__ RawDims<DPL> load_raw(const uint16_t* p) {
-  RawDims<DPL> r;
-  if constexpr (DPL == 4) {
-    const uint2 v = __ldg(reinterpret_cast<const uint2*>(p));
-    r.w[0] = v.x;
-    r.w[1] = v.y;
-  } else {
-    r.w[0] = __ldg(reinterpret_cast<const uint32_t*>(p));
-  }
-  return r;
-}
 
 template <int DPL>
 __device__ __forceinline__ void unpack(const RawDims<DPL>& r, float* out) {
@@ -68,20 +54,49 @@ __device__ __forceinline__ int64_t kept_prefix(const DecodeArgs& a, int s) {
 }
 
 constexpr int kDecWarps = 4;       // consumer warps per CTA
-constexpr int kStages = 4;         // shared-memory stages of cache rows
-constexpr int kStageRows = 32;     // rows per stage (8 per consumer warp)
+constexpr int kStages = 2;         // shared-memory stages of cache rows
+constexpr int kTileRows = 16;      // rows of one MMA tile (one consumer warp)
+constexpr int kStageRows = kDecWarps * kTileRows;
 constexpr int kDecThreads = (kDecWarps + 1) * 32;   // + one producer warp
 
-__host__ __device__ constexpr int decode_smem_bytes(int d) { return 2 * kStages * kStageRows * d * 2; }
+// K rows sit 16 bytes apart beyond their length, so that the eight rows read
+// by one fragment load fall in different banks; V rows are packed.
+__host__ __device__ constexpr int k_stride_bytes(int d) { return 2 * d + 16; }
+__host__ __device__ constexpr int decode_smem_bytes(int d) {
+  return kStages * kStageRows * (k_stride_bytes(d) + 2 * d);
+}
 
+__device__ __forceinline__ uint32_t lds32(const uint8_t* p) { return *reinterpret_cast<const uint32_t*>(p); }
+
+// D = A B + D for one 16 x 8 x 16 bf16 tile (fp32 accumulate): A = 16 cache
+// rows x 16 dims, B = 16 dims x 8 query heads.
+__device__ __forceinline__ void mma16816(float* c, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+      "{%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// Consumer warps: q . k for 16 rows x 8 (padded) heads on the tensor cores,
+// in the fragment layout (lane = 4 g + t holds rows g and g + 8 of heads 2t
+// and 2t + 1); the online softmax runs there; the probabilities and rescale
+// factors then go through a small per-warp shared buffer to the output
+// accumulation, where the lanes run over the head dimension (DPL each).
 template <int DPL, int GM>
 __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const DecodeArgs a) {
-  constexpr int RB = GM <= 4 ? kRowBatch : kRowBatch / 2;   // rows per batch (registers)
+  constexpr int D = DPL * 32;
+  constexpr int KS = D / 16;                                // MMA k-steps
+  constexpr int KSTR = k_stride_bytes(D);
+  constexpr int VSTR = 2 * D;
   extern __shared__ __align__(128) uint8_t stage_mem[];     // K stages, then V stages
   __shared__ uint64_t full_bar[kStages], empty_bar[kStages];
   __shared__ int abort_flag;
   __shared__ float red[kDecWarps][GM][2];                   // per-warp (max2, sum) per head
-  __shared__ float racc[kDecWarps][GM][128];
+  __shared__ __align__(16) float pbuf[kDecWarps][kTileRows][8];
+  __shared__ __align__(16) float fbuf[kDecWarps][8];
+  __shared__ float okbuf[kDecWarps][kTileRows];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int u = blockIdx.x / a.n_splits;
   const int split = blockIdx.x % a.n_splits;
@@ -103,11 +118,10 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const Decod
   if (r0 >= m) return;                              // (uniform: no partial is read)
   const int r1 = (m - r0 < a.rows_per_split) ? m : r0 + a.rows_per_split;
   const int nst = (r1 - r0 + kStageRows - 1) / kStageRows;
-  const int rowbytes = a.d * 2;
   const int64_t kb = l * a.k_layer + (a.varlen ? row0 * a.k_tok : s * a.k_seq) + h * a.k_head;
   const int64_t vb = l * a.v_layer + (a.varlen ? row0 * a.v_tok : s * a.v_seq) + h * a.v_head;
   uint8_t* ks = stage_mem;
-  uint8_t* vs = stage_mem + kStages * kStageRows * rowbytes;
+  uint8_t* vs = stage_mem + kStages * kStageRows * KSTR;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < kStages; ++i) {
@@ -119,18 +133,19 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const Decod
   }
   __syncthreads();
 
-  float mx[GM], sum[GM], acc[GM][DPL];
+  // fragment-layout state: heads 2t, 2t+1 of this lane's rows
+  const int g = lane >> 2, t = lane & 3;
+  float mx[2] = {-INFINITY, -INFINITY}, sm[2] = {0.f, 0.f};
+  // output accumulators: lanes over dims
+  float2 acc[GM][DPL / 2];
 #pragma unroll
-  for (int g = 0; g < GM; ++g) {
-    mx[g] = -INFINITY;
-    sum[g] = 0.f;
+  for (int hh = 0; hh < GM; ++hh)
 #pragma unroll
-    for (int i = 0; i < DPL; ++i) acc[g][i] = 0.f;
-  }
+    for (int i = 0; i < DPL / 2; ++i) acc[hh][i] = make_float2(0.f, 0.f);
 
   if (warp == kDecWarps) {
     // ---------------------------------------------------------- producer
-    const bool kc = a.k_tok == a.d, vc = a.v_tok == a.d;   // rows contiguous
+    const bool vc = a.v_tok == D;                   // V rows contiguous
     int issued = 0;
     for (int st = 0; st < nst; ++st) {
       const int slot = st % kStages;
@@ -139,19 +154,17 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const Decod
       if (!__shfl_sync(0xffffffffu, static_cast<int>(ok), 0)) break;
       const int rs = r0 + st * kStageRows;
       const int nr = (r1 - rs < kStageRows) ? r1 - rs : kStageRows;
-      if (lane == 0) mbar_arrive_expect_tx(&full_bar[slot], static_cast<uint32_t>(2 * nr * rowbytes));
+      if (lane == 0) mbar_arrive_expect_tx(&full_bar[slot], static_cast<uint32_t>(2 * nr * VSTR));
       __syncwarp();
-      uint8_t* kd = ks + slot * kStageRows * rowbytes;
-      uint8_t* vd = vs + slot * kStageRows * rowbytes;
-      if (kc) {
-        if (lane == 0) bulk_copy_g2s(kd, a.k + kb + static_cast<int64_t>(rs) * a.k_tok, nr * rowbytes, &full_bar[slot]);
-      } else if (lane < nr) {
-        bulk_copy_g2s(kd + lane * rowbytes, a.k + kb + static_cast<int64_t>(rs + lane) * a.k_tok, rowbytes, &full_bar[slot]);
-      }
+      uint8_t* kd = ks + slot * kStageRows * KSTR;
+      uint8_t* vd = vs + slot * kStageRows * VSTR;
+      for (int r = lane; r < nr; r += 32)
+        bulk_copy_g2s(kd + r * KSTR, a.k + kb + static_cast<int64_t>(rs + r) * a.k_tok, VSTR, &full_bar[slot]);
       if (vc) {
-        if (lane == 0) bulk_copy_g2s(vd, a.v + vb + static_cast<int64_t>(rs) * a.v_tok, nr * rowbytes, &full_bar[slot]);
-      } else if (lane < nr) {
-        bulk_copy_g2s(vd + lane * rowbytes, a.v + vb + static_cast<int64_t>(rs + lane) * a.v_tok, rowbytes, &full_bar[slot]);
+        if (lane == 0) bulk_copy_g2s(vd, a.v + vb + static_cast<int64_t>(rs) * a.v_tok, nr * VSTR, &full_bar[slot]);
+      } else {
+        for (int r = lane; r < nr; r += 32)
+          bulk_copy_g2s(vd + r * VSTR, a.v + vb + static_cast<int64_t>(rs + r) * a.v_tok, VSTR, &full_bar[slot]);
       }
       ++issued;
     }
@@ -164,129 +177,160 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const Decod
     __syncwarp();
   } else {
     // --------------------------------------------------------- consumers
-    const int d0 = lane * DPL;
-    float q[GM][DPL];
+    // B fragments of the query heads (head g of the group, zero past G)
+    uint32_t qb[KS][2];
+    {
+      const uint16_t* qp = a.q + l * a.q_layer + s * a.q_seq + static_cast<int64_t>(h * G + (g < G ? g : 0)) * a.q_head;
 #pragma unroll
-    for (int g = 0; g < GM; ++g) {
-      const uint16_t* qp = a.q + l * a.q_layer + s * a.q_seq +
-                           static_cast<int64_t>(h * G + (g < G ? g : 0)) * a.q_head + d0;
-#pragma unroll
-      for (int i = 0; i < DPL; ++i) q[g][i] = g < G ? bf16f(qp[i]) * a.c1 : 0.f;
+      for (int k = 0; k < KS; ++k) {
+        qb[k][0] = g < G ? __ldg(reinterpret_cast<const uint32_t*>(qp + k * 16 + 2 * t)) : 0u;
+        qb[k][1] = g < G ? __ldg(reinterpret_cast<const uint32_t*>(qp + k * 16 + 2 * t + 8)) : 0u;
+      }
     }
     const int32_t* idx = nullptr;
     if (a.keep_idx != nullptr)
       idx = a.keep_idx + (a.varlen ? (static_cast<int64_t>(l) * a.Hkv + h) * a.Ktot + row0
                                    : static_cast<int64_t>(u) * a.K_dense);
+    const float c1 = a.c1;
+    const int d0 = lane * DPL;
+    float* pw = &pbuf[warp][0][0];
     for (int st = 0; st < nst; ++st) {
       const int slot = st % kStages;
       const bool got = mbar_wait(&full_bar[slot], (st / kStages) & 1, &abort_flag, a.status);
       if (!__all_sync(0xffffffffu, got)) break;
-      const int rs = r0 + st * kStageRows;
-      const uint8_t* kst = ks + slot * kStageRows * rowbytes + d0 * 2;
-      const uint8_t* vst = vs + slot * kStageRows * rowbytes + d0 * 2;
+      const int tr0 = r0 + st * kStageRows + warp * kTileRows;   // first row of this warp's tile
+      const uint8_t* kt = ks + slot * kStageRows * KSTR + warp * kTileRows * KSTR;
+      const uint8_t* vt = vs + slot * kStageRows * VSTR + warp * kTileRows * VSTR;
+      if (tr0 < r1) {                                            // (uniform)
+        float c[4] = {0.f, 0.f, 0.f, 0.f};
+        const uint8_t* ka = kt + g * KSTR + 4 * t;
 #pragma unroll
-      for (int half = 0; half < kStageRows / kDecWarps / RB; ++half) {
-        const int jr0 = warp * (kStageRows / kDecWarps) + half * RB;   // row within the stage
-        RawDims<DPL> kraw[RB], vraw[RB];
-        bool ok[RB];
+        for (int k = 0; k < KS; ++k)
+          mma16816(c, lds32(ka + 32 * k), lds32(ka + 8 * KSTR + 32 * k), lds32(ka + 32 * k + 16),
+                   lds32(ka + 8 * KSTR + 32 * k + 16), qb[k][0], qb[k][1]);
+        // rows g and g + 8: inside the split, and a kept slot
+        const int ra = tr0 + g, rb = tr0 + g + 8;
+        const bool oka = ra < r1 && (idx == nullptr || __ldg(idx + ra) >= 0);
+        const bool okb = rb < r1 && (idx == nullptr || __ldg(idx + rb) >= 0);
+        const float s0 = oka ? c[0] * c1 : -INFINITY, s1 = oka ? c[1] * c1 : -INFINITY;
+        const float s2 = okb ? c[2] * c1 : -INFINITY, s3 = okb ? c[3] * c1 : -INFINITY;
+        float tm0 = fmaxf(s0, s2), tm1 = fmaxf(s1, s3);
 #pragma unroll
-        for (int j = 0; j < RB; ++j) {
-          const int r = rs + jr0 + j;
-          ok[j] = r < r1 && (idx == nullptr || __ldg(idx + (r < r1 ? r : r1 - 1)) >= 0);
-          kraw[j] = *reinterpret_cast<const RawDims<DPL>*>(kst + (jr0 + j) * rowbytes);
-          vraw[j] = *reinterpret_cast<const RawDims<DPL>*>(vst + (jr0 + j) * rowbytes);
+        for (int o = 4; o < 32; o <<= 1) {
+          tm0 = fmaxf(tm0, __shfl_xor_sync(0xffffffffu, tm0, o));
+          tm1 = fmaxf(tm1, __shfl_xor_sync(0xffffffffu, tm1, o));
         }
-        float sc[GM][RB];
-#pragma unroll
-        for (int j = 0; j < RB; ++j) {
-          float kr[DPL];
-          unpack<DPL>(kraw[j], kr);
-#pragma unroll
-          for (int g = 0; g < GM; ++g) {
-            float t = 0.f;
-#pragma unroll
-            for (int i = 0; i < DPL; ++i) t = fmaf(q[g][i], kr[i], t);
-            sc[g][j] = t;
+        const float mn0 = fmaxf(mx[0], tm0), mn1 = fmaxf(mx[1], tm1);
+        const float f0 = mn0 == -INFINITY ? 1.f : fast_exp2(mx[0] - mn0);
+        const float f1 = mn1 == -INFINITY ? 1.f : fast_exp2(mx[1] - mn1);
+        const float p0 = mn0 == -INFINITY ? 0.f : fast_exp2(s0 - mn0);
+        const float p1 = mn1 == -INFINITY ? 0.f : fast_exp2(s1 - mn1);
+        const float p2 = mn0 == -INFINITY ? 0.f : fast_exp2(s2 - mn0);
+        const float p3 = mn1 == -INFINITY ? 0.f : fast_exp2(s3 - mn1);
+        sm[0] = sm[0] * f0 + (p0 + p2);
+        sm[1] = sm[1] * f1 + (p1 + p3);
+        mx[0] = mn0;
+        mx[1] = mn1;
+        *reinterpret_cast<float2*>(pw + g * 8 + 2 * t) = make_float2(p0, p1);
+        *reinterpret_cast<float2*>(pw + (g + 8) * 8 + 2 * t) = make_float2(p2, p3);
+        if (g == 0) *reinterpret_cast<float2*>(&fbuf[warp][2 * t]) = make_float2(f0, f1);
+        if (t == 0) {
+          okbuf[warp][g] = oka ? 1.f : 0.f;
+          okbuf[warp][g + 8] = okb ? 1.f : 0.f;
+        }
+        __syncwarp();
+        // o_h = o_h f_h + sum_j p_hj v_j, lanes over dims
+        {
+          const float4 F0 = *reinterpret_cast<const float4*>(&fbuf[warp][0]);
+          float F[8] = {F0.x, F0.y, F0.z, F0.w, 1.f, 1.f, 1.f, 1.f};
+          if (GM > 4) {
+            const float4 F1 = *reinterpret_cast<const float4*>(&fbuf[warp][4]);
+            F[4] = F1.x; F[5] = F1.y; F[6] = F1.z; F[7] = F1.w;
           }
+#pragma unroll
+          for (int hh = 0; hh < GM; ++hh)
+#pragma unroll
+            for (int i = 0; i < DPL / 2; ++i) acc[hh][i] = __fmul2_rn(acc[hh][i], make_float2(F[hh], F[hh]));
         }
+        const bool all_ok = __all_sync(0xffffffffu, oka && okb);
+#pragma unroll 4
+        for (int j = 0; j < kTileRows; ++j) {
+          float vr[DPL];
+          unpack<DPL>(*reinterpret_cast<const RawDims<DPL>*>(vt + j * VSTR + d0 * 2), vr);
+          // rows past the end hold stale shared memory: their values are
+          // zeroed (a weight of zero would not remove a stale NaN)
+          if (!all_ok) {
+            const bool okj = okbuf[warp][j] != 0.f;
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-          for (int g = 0; g < GM; ++g)
-            if (g < G) {
-#pragma unroll
-              for (int j = 0; j < RB; ++j) sc[g][j] += __shfl_xor_sync(0xffffffffu, sc[g][j], o);
-            }
-        // rows past the end hold stale shared memory: their values are
-        // zeroed (a weight of zero would not remove a stale NaN)
-        float vr[RB][DPL];
-#pragma unroll
-        for (int j = 0; j < RB; ++j) {
-          unpack<DPL>(vraw[j], vr[j]);
-#pragma unroll
-          for (int i = 0; i < DPL; ++i) vr[j][i] = ok[j] ? vr[j][i] : 0.f;
-        }
-#pragma unroll
-        for (int g = 0; g < GM; ++g) {
-          if (g >= G) continue;
-          float bm = -INFINITY;
-#pragma unroll
-          for (int j = 0; j < RB; ++j) {
-            if (!ok[j]) sc[g][j] = -INFINITY;
-            bm = fmaxf(bm, sc[g][j]);
+            for (int i = 0; i < DPL; ++i) vr[i] = okj ? vr[i] : 0.f;
           }
-          if (bm == -INFINITY) continue;            // (uniform) nothing valid here
-          const float mn = fmaxf(mx[g], bm);
-          const float rescale = fast_exp2(mx[g] - mn);
-          sum[g] *= rescale;
-#pragma unroll
-          for (int i = 0; i < DPL; ++i) acc[g][i] *= rescale;
-#pragma unroll
-          for (int j = 0; j < RB; ++j) {
-            const float p = ok[j] ? fast_exp2(sc[g][j] - mn) : 0.f;
-            sum[g] += p;
-#pragma unroll
-            for (int i = 0; i < DPL; ++i) acc[g][i] = fmaf(p, vr[j][i], acc[g][i]);
+          const float4 P0 = *reinterpret_cast<const float4*>(pw + j * 8);
+          float P[8] = {P0.x, P0.y, P0.z, P0.w, 0.f, 0.f, 0.f, 0.f};
+          if (GM > 4) {
+            const float4 P1 = *reinterpret_cast<const float4*>(pw + j * 8 + 4);
+            P[4] = P1.x; P[5] = P1.y; P[6] = P1.z; P[7] = P1.w;
           }
-          mx[g] = mn;
+#pragma unroll
+          for (int hh = 0; hh < GM; ++hh)
+#pragma unroll
+            for (int i = 0; i < DPL / 2; ++i)
+              acc[hh][i] = __ffma2_rn(make_float2(P[hh], P[hh]), make_float2(vr[2 * i], vr[2 * i + 1]), acc[hh][i]);
         }
+        __syncwarp();                                              // pbuf is rewritten next tile
       }
-      __syncwarp();
       if (lane == 0) mbar_arrive(&empty_bar[slot]);
     }
-    // this warp's state per head, for the merge
+    // per-head sums over the lanes of a head column (g = 0..7)
 #pragma unroll
-    for (int g = 0; g < GM; ++g) {
-      if (lane == 0) {
-        red[warp][g][0] = mx[g];
-        red[warp][g][1] = sum[g];
-      }
-#pragma unroll
-      for (int i = 0; i < DPL; ++i) racc[warp][g][d0 + i] = acc[g][i];
+    for (int o = 4; o < 32; o <<= 1) {
+      sm[0] += __shfl_xor_sync(0xffffffffu, sm[0], o);
+      sm[1] += __shfl_xor_sync(0xffffffffu, sm[1], o);
     }
+    if (g == 0) {
+      if (2 * t < GM) {
+        red[warp][2 * t][0] = mx[0];
+        red[warp][2 * t][1] = sm[0];
+      }
+      if (2 * t + 1 < GM) {
+        red[warp][2 * t + 1][0] = mx[1];
+        red[warp][2 * t + 1][1] = sm[1];
+      }
+    }
+  }
+  __syncthreads();   // every stage consumed, every copy landed: the stages are free
+  float* racc = reinterpret_cast<float*>(stage_mem);          // [warp][head][D]
+  if (warp < kDecWarps) {
+    const int d0 = lane * DPL;
+#pragma unroll
+    for (int hh = 0; hh < GM; ++hh)
+#pragma unroll
+      for (int i = 0; i < DPL / 2; ++i) {
+        racc[(warp * GM + hh) * D + d0 + 2 * i] = acc[hh][i].x;
+        racc[(warp * GM + hh) * D + d0 + 2 * i + 1] = acc[hh][i].y;
+      }
   }
   __syncthreads();
   if (warp < kDecWarps) {
     const int d0 = lane * DPL;
-    for (int g = warp; g < G; g += kDecWarps) {
+    for (int gg = warp; gg < G; gg += kDecWarps) {
       float M = -INFINITY;
 #pragma unroll
-      for (int w = 0; w < kDecWarps; ++w) M = fmaxf(M, red[w][g][0]);
+      for (int w = 0; w < kDecWarps; ++w) M = fmaxf(M, red[w][gg][0]);
       float L = 0.f, o[DPL];
 #pragma unroll
       for (int i = 0; i < DPL; ++i) o[i] = 0.f;
       if (M > -INFINITY) {
 #pragma unroll
         for (int w = 0; w < kDecWarps; ++w) {
-          const float mw = red[w][g][0];
+          const float mw = red[w][gg][0];
           if (mw == -INFINITY) continue;
           const float f = exp2f(mw - M);
-          L += f * red[w][g][1];
+          L += f * red[w][gg][1];
 #pragma unroll
-          for (int i = 0; i < DPL; ++i) o[i] += f * racc[w][g][d0 + i];
+          for (int i = 0; i < DPL; ++i) o[i] += f * racc[(w * GM + gg) * D + d0 + i];
         }
       }
-      float* out = a.part + ((static_cast<int64_t>(u) * a.n_splits + split) * a.G + g) * (a.d + 2);
+      float* out = a.part + ((static_cast<int64_t>(u) * a.n_splits + split) * a.G + gg) * (a.d + 2);
 #pragma unroll
       for (int i = 0; i < DPL; ++i) out[d0 + i] = o[i];
       if (lane == 0) {
@@ -360,6 +404,10 @@ cudaError_t launch_decode_d(const DecodeArgs& a, cudaStream_t stream) {
   const unsigned grid2 = static_cast<unsigned>((warps2 * 32 + 255) / 256);
   const int smem = decode_smem_bytes(a.d);
   cudaError_t e;
+  if (grid1 == 0) {                                  // no rows anywhere: the merge writes zeros
+    decode_combine_kernel<DPL><<<grid2, 256, 0, stream>>>(a);
+    return cudaGetLastError();
+  }
   if (a.G <= 4) {
     e = cudaFuncSetAttribute(decode_partial_kernel<DPL, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;

@@ -656,7 +656,17 @@ int role_alloc_select(const rolekv_batch* batch, const float* scores, const uint
 }
 
 namespace {
-constexpr int kDecodeRowsPerSplit = 512;
+constexpr int kDecodeRowsPerSplit = 1024;
+
+// Splits of at most kDecodeRowsPerSplit rows, equal in length and a multiple
+// of the kernel's 64-row stage, so that a unit's splits finish together.
+void decode_split(int64_t m_max, int32_t* rows_per_split, int32_t* n_splits) {
+  const int64_t ns = m_max > 0 ? (m_max + kDecodeRowsPerSplit - 1) / kDecodeRowsPerSplit : 1;
+  int64_t r = (m_max + ns - 1) / ns;
+  r = r > 0 ? (r + 63) / 64 * 64 : 64;
+  *rows_per_split = static_cast<int32_t>(r);
+  *n_splits = static_cast<int32_t>((m_max + r - 1) / r);
+}
 
 // Rows of the largest sequence and the packed row total at this budget.
 void decode_rows(const BatchInfo& bi, const rolekv_batch* bt, int64_t bfx, int64_t* m_max,
@@ -676,7 +686,8 @@ void decode_rows(const BatchInfo& bi, const rolekv_batch* bt, int64_t bfx, int64
 }
 
 size_t decode_ws_bytes(const BatchInfo& bi, int64_t m_max) {
-  const int64_t splits = (m_max + kDecodeRowsPerSplit - 1) / kDecodeRowsPerSplit;
+  int32_t rps, splits;
+  decode_split(m_max, &rps, &splits);
   return static_cast<size_t>(bi.n_units) * static_cast<size_t>(splits > 0 ? splits : 1) * bi.G *
          (bi.d + 2) * sizeof(float);
 }
@@ -753,8 +764,7 @@ int decode_attention(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k
   a.v_tok = v_cache.s_tok;
   a.keep_idx = keep_idx;
   a.c1 = (scale > 0.f ? scale : 1.0f / std::sqrt(static_cast<float>(bi.d))) * 1.4426950408889634f;
-  a.rows_per_split = kDecodeRowsPerSplit;
-  a.n_splits = static_cast<int32_t>((m_max + kDecodeRowsPerSplit - 1) / kDecodeRowsPerSplit);
+  decode_split(m_max, &a.rows_per_split, &a.n_splits);
   a.part = static_cast<float*>(workspace);
   a.out = out;
   a.o_seq = static_cast<int64_t>(bi.Hq) * bi.d;

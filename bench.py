@@ -207,7 +207,8 @@ def run_gpu(args):
     roles = torch.as_tensor(roles_np, device=dev)
     batch = R.Batch(w.L, w.b, w.Hq, w.Hkv, w.d, w.n, seqlens=list(w.seqlens) if w.varlen else None,
                     device=dev)
-    policy = {"quota": R.POLICY_ROLE_QUOTA, "global": R.POLICY_GLOBAL, "fair": R.POLICY_FAIR}[args.policy]
+    policy = {"quota": R.POLICY_ROLE_QUOTA, "global": R.POLICY_GLOBAL, "fair": R.POLICY_FAIR,
+              "slack": R.POLICY_SLACK}[args.policy]
     params = R.select_params(B, I.PAPER_ALPHA, alpha_key=0.0, key_role=I.ROLE_KEY, policy=policy,
                              keep_last=args.keep_last)
     scores = torch.empty(batch.score_shape(), dtype=torch.float32, device=dev)
@@ -527,7 +528,7 @@ def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_o
 
 # ------------------------------------------------------ CPU oracle baseline --
 
-POLICY_CODES = {"quota": 0, "global": 1, "fair": 2}
+POLICY_CODES = {"quota": 0, "global": 1, "fair": 2, "slack": 3}
 
 
 def oracle_units(w, B, units, qw_bits, k_bits, v_bits, roles_np, policy="quota", keep_last=0,
@@ -682,8 +683,9 @@ def main(argv=None):
     ap.add_argument("--score", choices=["snapkv", "quest"], default="snapkv",
                     help="score of the SnapKV workloads: windowed mass, or the Quest page bound")
     ap.add_argument("--page", type=int, default=16, help="tokens per page of the Quest bound")
-    ap.add_argument("--policy", choices=["quota", "global", "fair"], default="quota",
-                    help="budget split: role quotas (the method), plain top-k, or fair eviction")
+    ap.add_argument("--policy", choices=["quota", "global", "fair", "slack"], default="quota",
+                    help="budget split: role quotas (the method), plain top-k, fair eviction, or "
+                         "role quotas with the slack of saturated buckets filled by score")
     ap.add_argument("--keep-last", type=int, default=0,
                     help="recency floor: always keep each sequence's last tokens")
     ap.add_argument("--layers", type=int, default=0,

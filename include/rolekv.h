@@ -75,6 +75,7 @@ extern "C" {
 #define ROLEKV_POLICY_ROLE_QUOTA 0  /* the combined method (Section 4.1)       */
 #define ROLEKV_POLICY_GLOBAL 1      /* plain top-k, optional role ban (Sec. 4) */
 #define ROLEKV_POLICY_FAIR 2        /* equal retention rate per role (Sec. 5)  */
+#define ROLEKV_POLICY_SLACK 3       /* slack of saturated buckets by score     */
 
 #define ROLEKV_MAX_ROLES 8
 #define ROLEKV_SELECT_MAX_N 40960   /* largest sequence role_alloc_select takes */
@@ -111,6 +112,13 @@ typedef struct rolekv_batch {
  *              ROLEKV_POLICY_FAIR: the fair-eviction baseline of Section 5
  *              (equal retention rate per role): as ROLE_QUOTA with every
  *              non-banned role weighted by its token count; alpha is unused.
+ *              ROLEKV_POLICY_SLACK: the other reading of Algorithm 1's
+ *              "redistribute unused budget from saturated buckets": one
+ *              round of the ROLE_QUOTA split (no water-filling), each quota
+ *              capped at its bucket's size, then the slots that saturated
+ *              buckets leave go to the highest-scoring tokens of the
+ *              eligible buckets not kept yet (ties to the lower index); the
+ *              total is the same min(ceil(B*n), eligible tokens).
  *   ban_mask   bit r set: role r keeps nothing.
  *   keep_last  recency floor (SnapKV's observation window, Section 7): the
  *              last R = min(keep_last, n, ceil(B*n)) tokens of each sequence

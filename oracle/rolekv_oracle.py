@@ -29,10 +29,12 @@ matmul / sort as the only library steps:
                            top-ceil(alpha_r B n_kv) per role bucket, alpha
                            renormalised over buckets, slack from saturated
                            buckets redistributed (Section 4.1; Algorithm 1).
-                           Two more splits: GLOBAL (plain top-k, optional
-                           role ban; Sections 2 and 4) and FAIR (equal
+                           Three more splits: GLOBAL (plain top-k, optional
+                           role ban; Sections 2 and 4), FAIR (equal
                            retention rate per role; Section 5
-                           "Fair-eviction baseline").
+                           "Fair-eviction baseline") and SLACK (the slack of
+                           saturated buckets filled by score instead of
+                           in proportion to alpha).
 * ``select_unit``       -- per-bucket top-q_r by pooled score (Algorithm 1);
                            ``select_batch`` optionally keeps the last R
                            tokens first (SnapKV's recency floor, Section 7).
@@ -65,6 +67,7 @@ FIXED_ONE = 1_000_000  # fixed-point unit for budgets and alphas (6 decimals)
 POLICY_ROLE_QUOTA = 0
 POLICY_GLOBAL = 1
 POLICY_FAIR = 2
+POLICY_SLACK = 3
 
 
 # ----------------------------------------------------------------------------
@@ -254,6 +257,13 @@ def role_quotas(counts: Sequence[int], alpha: Sequence[float], budget: float, n:
     non-banned role equal to its token count, so each role keeps the same
     fraction of its tokens up to integer rounding; alpha is not used.
 
+    SLACK (the other reading of Algorithm 1's "redistribute unused budget
+    from saturated buckets"): one round of the ROLE_QUOTA split without the
+    water-filling, each quota capped at its bucket's size; the quotas then
+    sum to K minus the slack that saturated buckets leave, and select_batch
+    fills that slack with the best-scoring remaining tokens of the eligible
+    buckets.
+
     k_full, when given, replaces ceil(B n) as the budget to split (the
     recency floor of select_batch takes its tokens out of it first).
     """
@@ -275,7 +285,7 @@ def role_quotas(counts: Sequence[int], alpha: Sequence[float], budget: float, n:
     S = [r for r in range(R) if a[r] > 0 and counts[r] > 0]
     K = min(K_full, sum(counts[r] for r in S))
     k_left = K
-    while S:
+    while S and policy != POLICY_SLACK:
         A = sum(a[r] for r in S)
         saturated = [r for r in S if a[r] * k_left >= counts[r] * A]
         if not saturated:
@@ -293,7 +303,18 @@ def role_quotas(counts: Sequence[int], alpha: Sequence[float], budget: float, n:
         left = k_left - sum(q[r] for r in S)
         for r in sorted(S, key=lambda r: (-rem[r], r))[:left]:
             q[r] += 1
+    if policy == POLICY_SLACK:
+        q = [min(q[r], counts[r]) for r in range(R)]
     return q
+
+
+def eligible_roles(counts: Sequence[int], alpha: Sequence[float], policy: int,
+                   ban_mask: int) -> list[int]:
+    """Roles whose bucket takes part in the split: not banned, holding tokens
+    and, for the alpha-weighted policies, alpha_r > 0."""
+    R = len(counts)
+    return [r for r in range(R) if counts[r] > 0 and not (ban_mask >> r) & 1
+            and (policy in (POLICY_GLOBAL, POLICY_FAIR) or to_fixed(alpha[r]) > 0)]
 
 
 def bucket_of_tokens(roles: np.ndarray, policy: int, ban_mask: int) -> np.ndarray:
@@ -467,6 +488,18 @@ def select_batch(batch: Batch, unit_scores: dict, roles, n_roles: int, alpha: Se
         bk = bucket_of_tokens(r, policy, ban_mask)
         bk[nf:] = -1
         idx = select_unit(np.asarray(sc, dtype=np.float64), bk, q)
+        if policy == POLICY_SLACK:
+            # the slack of saturated buckets goes to the best-scoring tokens
+            # of eligible buckets not kept yet (ties to the lower index)
+            E = eligible_roles(counts, al, policy, ban_mask)
+            K = min(width - forced, sum(counts[x] for x in E))
+            slack = K - sum(q)
+            if slack > 0:
+                sc64 = np.asarray(sc, dtype=np.float64)
+                pool = np.nonzero(np.isin(r[:nf], E))[0]
+                pool = np.setdiff1d(pool, idx)
+                order = np.lexsort((pool, -sc64[pool]))
+                idx = np.concatenate([idx, pool[order[:slack]]])
         idx = np.sort(np.concatenate([idx, np.arange(nf, n, dtype=np.int64)]))
         padded = np.full(width, -1, dtype=np.int64)
         padded[:idx.shape[0]] = idx

@@ -390,7 +390,7 @@ int fill_select(const BatchInfo& bi, const rolekv_batch* bt, const rolekv_select
   if (!(sp->budget > 0.f) || sp->budget > 1.f)
     return fail(ROLEKV_ERR_INVALID_ARG, "budget %g outside (0, 1]", static_cast<double>(sp->budget));
   if (sp->policy != ROLEKV_POLICY_ROLE_QUOTA && sp->policy != ROLEKV_POLICY_GLOBAL &&
-      sp->policy != ROLEKV_POLICY_FAIR)
+      sp->policy != ROLEKV_POLICY_FAIR && sp->policy != ROLEKV_POLICY_SLACK)
     return fail(ROLEKV_ERR_INVALID_ARG, "unknown policy %d", sp->policy);
   if (sp->keep_last < 0) return fail(ROLEKV_ERR_INVALID_ARG, "keep_last=%d must be >= 0", sp->keep_last);
   if (sp->key_role >= sp->n_roles) return fail(ROLEKV_ERR_INVALID_ARG, "key_role %d >= n_roles", sp->key_role);

@@ -116,6 +116,8 @@ struct SelShared {
   int32_t any_threshold;
   int32_t general;         // take the full-pass descent
   uint32_t partial_ties;   // buckets with more threshold ties than slots left
+  int32_t slack;           // SLACK policy: slots left to fill by score
+  uint32_t elig_mask;      // roles taking part in the split (bit r)
 };
 
 // Slots 4g .. 4g+3 of a score row; slots outside [off, off + n) read -inf.
@@ -247,9 +249,13 @@ __device__ void quotas_warp(const SelectArgs& a, int lane, int64_t K_full, SelSh
     }
   } else {
     bool live = valid && alpha > 0 && cnt > 0;
+    const unsigned elig_bits = __ballot_sync(0xffffffffu, live) & 0xFFu;
     const int64_t elig = sum8(live ? cnt : 0);
-    int64_t left = K_full < elig ? K_full : elig;
-    for (int it = 0; it <= kR; ++it) {
+    const int64_t k_all = K_full < elig ? K_full : elig;
+    int64_t left = k_all;
+    // SLACK: one round of the split, no water-filling (the slack of saturated
+    // buckets is filled by score afterwards)
+    for (int it = 0; it <= kR && a.policy != ROLEKV_POLICY_SLACK; ++it) {
       const int64_t A = sum8(live ? alpha : 0);
       if (A == 0) break;
       const bool sat = live && alpha * left >= cnt * A;
@@ -275,6 +281,14 @@ __device__ void quotas_warp(const SelectArgs& a, int lane, int64_t K_full, SelSh
       if (lx && (rx > rem || (rx == rem && x < r))) ++rank;
     }
     if (live && A != 0 && rank < extra) q += 1;
+    if (a.policy == ROLEKV_POLICY_SLACK) {
+      q = q < cnt ? q : cnt;
+      const int64_t slack = k_all - sum8(q);
+      if (lane == 0) {
+        S.slack = static_cast<int32_t>(slack);
+        S.elig_mask = elig_bits;
+      }
+    }
     bsize = cnt;
   }
   int mode = 0;
@@ -530,6 +544,8 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
     S.general = 0;
     S.top_and = 0xFFFFFFFFu;
     S.top_or = 0u;
+    S.slack = 0;
+    S.elig_mask = 0u;
   }
   for (int x = tid; x < kR * 256; x += NT) (&S.hist[0][0])[x] = 0;
   {
@@ -890,9 +906,98 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
     }
   }
 
+  // ---- SLACK: the slots saturated buckets left go to the best-scoring
+  // tokens of eligible roles not kept yet (ties to the lower index): four
+  // 8-bit rounds over all slots for the slack-th largest such key, in the
+  // state of bucket 0, whose own selection is complete.
+  if (S.slack > 0) {
+    const uint32_t elig = S.elig_mask;
+    auto candidate = [&](uint32_t rw, uint32_t fb, int g, int j) {
+      const uint32_t r = (rw >> (8 * j)) & 0xFFu;
+      const int slot = 4 * g + j;
+      return r < static_cast<uint32_t>(kR) && ((elig >> r) & 1u) && !((fb >> j) & 1u) &&
+             !((bits[slot >> 5] >> (slot & 31)) & 1u);
+    };
+    if (tid == 0) {
+      S.prefix[0] = 0;
+      S.need[0] = S.slack;
+      S.partial_ties = 0;
+    }
+    for (int x = tid; x < 256; x += NT) S.hist[0][x] = 0;
+    __syncthreads();
+    for (int round = 0; round < 4; ++round) {
+      const int shift = 24 - 8 * round;
+      for (int i = 0; i < iters; ++i) {
+        const int g = i * NT + tid;
+        if (g >= ngroups) break;
+        const uint4 kv = keys4[g];
+        const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
+        const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
+        const uint32_t fb = floor_bits(4 * g - off, v.nf, n);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          if (!candidate(rw, fb, g, j)) continue;
+          if (round > 0 && (kk[j] >> (shift + 8)) != (S.prefix[0] >> (shift + 8))) continue;
+          atomicAdd(&S.hist[0][(kk[j] >> shift) & 0xFFu], 1);
+        }
+      }
+      __syncthreads();
+      if (warp == 0) descend(S, 0, lane, shift);
+      __syncthreads();
+    }
+    // candidates above the threshold join; the rest of the ties in index order
+    const uint32_t T = S.thr[0], P = S.prefix[0];
+    const int need = S.need[0];
+    const bool partial = S.partial_ties & 1u;
+    __syncthreads();
+    for (int i = 0; i < iters; ++i) {
+      const int g = i * NT + tid;
+      if (g >= ngroups) break;
+      const uint4 kv = keys4[g];
+      const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
+      const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
+      const uint32_t fb = floor_bits(4 * g - off, v.nf, n);
+      uint32_t m4 = 0;
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (kk[j] >= T && candidate(rw, fb, g, j)) m4 |= 1u << j;
+      if (m4) atomicOr(&bits[g >> 3], m4 << (4 * (g & 7)));
+    }
+    __syncthreads();
+    if (partial) {
+      auto tie_mask = [&](int q) {
+        uint32_t mk = 0;
+#pragma unroll
+        for (int gg = 0; gg < 8; ++gg) {
+          const int g = 8 * q + gg;
+          if (g >= ngroups) break;
+          const uint4 kv = keys4[g];
+          const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
+          const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
+          const uint32_t fb = floor_bits(4 * g - off, v.nf, n);
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            if (kk[j] == P && candidate(rw, fb, g, j)) mk |= 1u << (4 * gg + j);
+        }
+        return mk;
+      };
+      scan_words<NT>(nwords, tie_mask, [&](int q, uint32_t mk, int rank) {
+        uint32_t keepm = 0;
+        while (mk != 0 && rank < need) {
+          const uint32_t low = mk & (0u - mk);
+          keepm |= low;
+          mk ^= low;
+          ++rank;
+        }
+        if (keepm) bits[q] |= keepm;
+      }, S.warp_tot);
+    }
+  }
+
   // ---- kept positions in ascending order
   int32_t* dst = a.keep_idx + S.keep_off;
-  const bool count_roles = a.kept_per_role != nullptr && a.policy == ROLEKV_POLICY_GLOBAL;
+  const bool count_roles = a.kept_per_role != nullptr &&
+                           (a.policy == ROLEKV_POLICY_GLOBAL || a.policy == ROLEKV_POLICY_SLACK);
   uint64_t kr = 0;
   const int total = scan_words<NT>(nwords, [&](int q) { return bits[q]; }, [&](int q, uint32_t m, int pos) {
     while (m != 0) {

@@ -18,7 +18,7 @@ _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "librolekv.
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA = 0, 1, 2, 3, 4
 STATUS_NONFINITE, STATUS_BAD_INDEX, STATUS_TIMEOUT = 1, 2, 4
-POLICY_ROLE_QUOTA, POLICY_GLOBAL, POLICY_FAIR = 0, 1, 2
+POLICY_ROLE_QUOTA, POLICY_GLOBAL, POLICY_FAIR, POLICY_SLACK = 0, 1, 2, 3
 MAX_ROLES = 8
 SELECT_MAX_N = 40960
 OP_SNAPKV, OP_H2O, OP_COMPRESS = 0, 1, 2

@@ -378,6 +378,76 @@ def pin_fair_quotas(O, rng):
     assert q == [25, 10, 15, 50]
 
 
+def pin_slack_fill(O, rng):
+    """SLACK (unused budget of saturated buckets filled by score): the quotas
+    are one round of the alpha split (exact rational shares, floors plus
+    largest remainders) capped at each bucket's size; when nothing saturates
+    the selection is ROLE_QUOTA's; on tiny units the tokens added beyond the
+    per-bucket top-q are the brute-force best subset of the remaining
+    eligible tokens, and a role with alpha 0 keeps nothing."""
+    for _ in range(300):
+        R = int(rng.integers(1, 7))
+        counts = [int(x) for x in rng.integers(0, 60, size=R)]
+        alpha = [float(x) for x in rng.choice([0.0, 0.02, 0.05, 0.2, 0.25, 0.7], size=R)]
+        n = sum(counts)
+        if n == 0:
+            continue
+        B = float(rng.choice([0.05, 0.1, 0.3, 0.5, 1.0]))
+        q = O.role_quotas(counts, alpha, B, n, policy=O.POLICY_SLACK)
+        a = {r: Fraction(round(alpha[r] * 1e6), 10**6) for r in range(R)}
+        E = [r for r in range(R) if a[r] > 0 and counts[r] > 0]
+        K = min(math.ceil(Fraction(round(B * 1e6), 10**6) * n), sum(counts[r] for r in E))
+        if not E:
+            assert q == [0] * R
+            continue
+        A = sum(a[r] for r in E)
+        share = {r: a[r] * K / A for r in E}
+        floors = {r: math.floor(share[r]) for r in E}
+        up = sorted(E, key=lambda r: (-(share[r] - floors[r]), r))[:K - sum(floors.values())]
+        for r in range(R):
+            want = min(counts[r], floors[r] + (1 if r in up else 0)) if r in E else 0
+            assert q[r] == want, (counts, alpha, B, q)
+        assert sum(q) <= K
+    # nothing saturates: the same keep set as the proportional split
+    b, n = 1, 400
+    batch = O.Batch(1, b, 1, 1, 8, n)
+    roles = np.repeat(np.arange(4, dtype=np.uint8), 100)[None, :]
+    sc = {0: rng.random(n)}
+    al = [0.25, 0.25, 0.25, 0.25]
+    same_q = O.select_batch(batch, sc, roles, 4, al, -1, 0.0, 0.2, O.POLICY_ROLE_QUOTA)[0][0]
+    same_s = O.select_batch(batch, sc, roles, 4, al, -1, 0.0, 0.2, O.POLICY_SLACK)[0][0]
+    assert np.array_equal(same_q, same_s)
+    for trial in range(30):
+        m = int(rng.integers(8, 14))
+        tb = O.Batch(1, 1, 1, 1, 8, m)
+        rl = rng.integers(0, 3, size=(1, m)).astype(np.uint8)
+        rl[0, 0] = 0                                    # role 0 is small: it saturates
+        rl[0, 1:] = np.where(rl[0, 1:] == 0, 1, rl[0, 1:])
+        sc = rng.integers(0, 5, size=m).astype(np.float64)
+        B = float(rng.choice([0.4, 0.5, 0.7]))
+        akey = float(rng.choice([0.0, 0.1]))
+        al = [0.8, 0.2, 0.0]                            # role 2 is the key role below
+        idx, per = O.select_batch(tb, {0: sc}, rl, 3, al, 2, akey, B, O.POLICY_SLACK)[0]
+        kept = [int(t) for t in idx if t >= 0]
+        counts = [int((rl[0] == x).sum()) for x in range(3)]
+        q = O.role_quotas(counts, [0.8, 0.2, akey], B, m, policy=O.POLICY_SLACK)
+        E = [x for x in range(3) if counts[x] > 0 and [0.8, 0.2, akey][x] > 0]
+        K = min(O.kept_count(m, B), sum(counts[x] for x in E))
+        assert len(kept) == K, (trial, kept, K)
+        base = set()
+        for r in range(3):
+            members = [t for t in range(m) if rl[0, t] == r]
+            best = min(((-sum(sc[list(sub)]), sub) for sub in itertools.combinations(members, q[r])))
+            base |= set(best[1])
+        assert base <= set(kept)
+        rest = [t for t in range(m) if rl[0, t] in E and t not in base]
+        extra = tuple(t for t in kept if t not in base)
+        best = min(((-sum(sc[list(sub)]), sub) for sub in itertools.combinations(rest, K - len(base))))
+        assert extra == best[1], (trial, extra, best)
+        if akey == 0.0:
+            assert per[2] == 0
+
+
 def pin_recency_floor(O, rng):
     """The recency floor keeps the last R = min(keep_last, n, ceil(B n))
     tokens and splits the other ceil(B n) - R slots over the earlier tokens:
@@ -482,5 +552,5 @@ ALL_PINS = [
     pin_two_level_scale, pin_window_covering_is_h2o, pin_gqa_grouping, pin_maxpool,
     pin_kept_count, pin_quota_golden, pin_quota_waterlevel, pin_key_ban,
     pin_global_is_full_sort, pin_bruteforce_select, pin_compact, pin_varlen_matches_dense,
-    pin_fair_quotas, pin_recency_floor, pin_quest_bound, pin_decode_attention,
+    pin_fair_quotas, pin_recency_floor, pin_quest_bound, pin_decode_attention, pin_slack_fill,
 ]

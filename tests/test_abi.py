@@ -99,7 +99,7 @@ def test_host_rejects_bad_arguments(lib):
     p_neg = R.select_params(0.1, [0.25, 0.0, -0.7, 0.05])
     rc = lib.role_alloc_select(ctypes.byref(b), f, f, ctypes.byref(p_neg), 1, f, None, None, None, None)
     assert rc == R.ERR_INVALID_ARG
-    p_pol = R.select_params(0.1, [0.25, 0.0, 0.7, 0.05], policy=3)
+    p_pol = R.select_params(0.1, [0.25, 0.0, 0.7, 0.05], policy=4)
     rc = lib.role_alloc_select(ctypes.byref(b), f, f, ctypes.byref(p_pol), 1, f, None, None, None, None)
     assert rc == R.ERR_INVALID_ARG                                      # unknown policy
     p_floor = R.select_params(0.1, [0.25, 0.0, 0.7, 0.05], keep_last=-1)

@@ -317,6 +317,12 @@ SELECT_CASES = [
     ("floor_over_budget", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=3001), 0.05, 0.0, 0, 0, 7, 1000),
     ("floor_fair_mid_n", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=12001), 0.10, 0.0, R.POLICY_FAIR, 0, 7, 64),
     ("floor_max_n", _w("long", L=1, b=1, Hq=4, Hkv=1, n=R.SELECT_MAX_N), 0.10, 0.0, 0, 0, 7, 64),
+    # role quotas with the slack of saturated buckets filled by score
+    ("slack_b50", _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=5000), 0.50, 0.02, R.POLICY_SLACK, 0, 7),
+    ("slack_b30_no_key_varlen", VARLEN4, 0.30, 0.0, R.POLICY_SLACK, 0, 7),
+    ("slack_floor_mid_n", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=12001), 0.20, 0.02, R.POLICY_SLACK, 0, 7, 64),
+    ("slack_ban_max_n", _w("long", L=1, b=1, Hq=4, Hkv=1, n=R.SELECT_MAX_N), 0.30, 0.02, R.POLICY_SLACK,
+     1 << I.ROLE_KEY, 1),
 ]
 
 

@@ -215,6 +215,18 @@ def _m_decode_unnormalised(O):
     _from_source(O, "return (e / e.sum(axis=1, keepdims=True)) @ vv", "return e @ vv", ["decode_attention"])
 
 
+def _m_slack_from_all_roles(O):
+    _from_source(O, "pool = np.nonzero(np.isin(r[:nf], E))[0]", "pool = np.arange(nf)", ["select_batch"])
+
+
+def _m_slack_waterfills(O):
+    _from_source(O, "while S and policy != POLICY_SLACK:", "while S:", ["role_quotas"])
+
+
+def _m_slack_not_filled(O):
+    _from_source(O, "if slack > 0:", "if slack > 10**9:", ["select_batch"])
+
+
 def _m_compact_off_by_one(O):
     orig = O.compact_unit
     O.compact_unit = lambda rows, idx: orig(rows, np.where(np.asarray(idx) >= 0, np.minimum(np.asarray(idx) + 1, rows.shape[0] - 1), -1))
@@ -226,7 +238,8 @@ MUTATIONS = [
     _m_round_not_ceil, _m_no_redistribution, _m_renormalise_all_buckets, _m_remainder_ties_high,
     _m_ties_to_high_index, _m_interleaved_gqa, _m_compact_off_by_one, _m_fair_uses_alpha,
     _m_floor_outside_budget, _m_floor_counts_whole_row, _m_quest_max_only, _m_quest_window_start,
-    _m_decode_keeps_padding, _m_decode_unnormalised,
+    _m_decode_keeps_padding, _m_decode_unnormalised, _m_slack_from_all_roles, _m_slack_waterfills,
+    _m_slack_not_filled,
 ]
 
 

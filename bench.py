@@ -65,6 +65,9 @@ def barrier(world: int):
         dist.barrier()
 
 
+HBM_NOMINAL_GBS = 7900.0   # GB300 HBM3e nominal bandwidth (context beside the measured peak)
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -325,6 +328,7 @@ def run_gpu(args):
                    "global_batch": world * w.b, "seq_len": w.n, "parallelism": f"replicas x{world}",
                    "l2": "inputs larger than L2, no flush"},
         "hbm_path_frac": path_frac,
+        "hbm_path_frac_nominal": counts["path_bytes"] / (ms_step / 1e3) / 1e9 / HBM_NOMINAL_GBS,
         "tensor_frac_of_measured_peak": tensor_util or None,
         "per_kernel_ms": per_kernel,
         "unit_tokens_per_s": world * w.L * w.Hkv * seq_tokens * args.steps / (elapsed_ms / 1e3),

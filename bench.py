@@ -595,13 +595,14 @@ def cpu_baseline(w, B, seconds: float, host_inputs, policy="quota", keep_last=0,
         t_total += time.perf_counter() - t0
         done += 1
         units.append(u)
-        if t_total >= seconds or done >= per_layer:
+        # layer 0's units, repeated if they take less than `seconds`
+        if t_total >= seconds or done >= 8 * per_layer:
             break
     seq_tokens = w.b * w.n if not w.varlen else sum(w.seqlens)
     value = (done / U) * seq_tokens / t_total
     return {"value": value, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
-            "sample": f"{done} of {U} (layer, sequence, KV head) units of layer 0, "
-                      f"{t_total:.1f} s, extrapolated linearly to the full step",
+            "sample": f"{done} unit passes over the {min(done, per_layer)} (sequence, KV head) units of "
+                      f"layer 0 (the step has {U}), {t_total:.1f} s, extrapolated linearly to the full step",
             "seconds": t_total}
 
 

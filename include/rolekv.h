@@ -42,6 +42,10 @@
  *   Varlen: [L][Hkv][Ktot], sequence s at offset cu_kept[s] = sum of K_s' for
  *   s' < s.  Kept positions are written in ascending order; when fewer than K_s
  *   tokens are eligible the tail of the row is -1.
+ * Batches without tokens.  When n_max is 0 or every sequence is empty, the
+ *   buffers sized by tokens or kept slots are empty and may be NULL; the
+ *   calls still write what is not empty: zero per-role kept counts and zero
+ *   decode outputs.
  * Ownership.  The caller owns every buffer; the library allocates, frees and
  *   synchronises nothing.  Every call enqueues work on `stream` (a
  *   cudaStream_t; NULL means the legacy default stream) and returns at once.

@@ -514,10 +514,11 @@ int snapkv_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k
   if (rc) return rc;
   if (pool_k < 1 || pool_k > 15 || pool_k % 2 == 0)
     return fail(ROLEKV_ERR_UNSUPPORTED, "pool_k=%d must be odd, 1..15", pool_k);
-  if (scores == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "scores is NULL");
   ScorePlan p;
   rc = plan_score(kModeSnapKV, bi, W, lse_win == nullptr, scores_prepool == nullptr, &p, true);
   if (rc) return rc;
+  if (bi.T == 0) return ROLEKV_OK;                 // no tokens: nothing to score
+  if (scores == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "scores is NULL");
   if ((rc = check_tensor("q_win", q_win, bi.d, bi.Hq, false, true))) return rc;
   if ((rc = check_tensor("k", k, bi.d, bi.Hkv, bi.varlen, true))) return rc;
   if ((rc = bind_workspace(p, workspace, workspace_bytes))) return rc;
@@ -544,10 +545,11 @@ int h2o_score(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k, float
   BatchInfo bi;
   int rc = check_batch(batch, &bi);
   if (rc) return rc;
-  if (scores == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "scores is NULL");
   ScorePlan p;
   rc = plan_score(kModeH2O, bi, 0, false, false, &p);
   if (rc) return rc;
+  if (bi.T == 0) return ROLEKV_OK;                 // no tokens: nothing to score
+  if (scores == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "scores is NULL");
   if ((rc = check_tensor("q", q, bi.d, bi.Hq, bi.varlen, true))) return rc;
   if ((rc = check_tensor("k", k, bi.d, bi.Hkv, bi.varlen, true))) return rc;
   if ((rc = bind_workspace(p, workspace, workspace_bytes))) return rc;
@@ -587,6 +589,7 @@ int quest_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k,
     return fail(ROLEKV_ERR_UNSUPPORTED, "head dim %d (quest_score takes 64 or 128)", bi.d);
   if (W < 1) return fail(ROLEKV_ERR_INVALID_ARG, "window W=%d must be >= 1", W);
   if (page < 1 || page > 4096) return fail(ROLEKV_ERR_INVALID_ARG, "page=%d outside 1..4096", page);
+  if (bi.T == 0) return ROLEKV_OK;                 // no tokens: nothing to score
   if (scores == nullptr || (reinterpret_cast<uintptr_t>(scores) & 3u))
     return fail(ROLEKV_ERR_INVALID_ARG, "scores must be a non-NULL, 4-byte aligned pointer");
   if ((rc = check_tensor("q_win", q_win, bi.d, bi.Hq, false, false))) return rc;
@@ -632,7 +635,7 @@ int role_alloc_select(const rolekv_batch* batch, const float* scores, const uint
   BatchInfo bi;
   int rc = check_batch(batch, &bi);
   if (rc) return rc;
-  if (scores == nullptr || roles == nullptr || keep_idx == nullptr)
+  if (bi.T > 0 && (scores == nullptr || roles == nullptr || keep_idx == nullptr))
     return fail(ROLEKV_ERR_INVALID_ARG, "scores, roles and keep_idx are required");
   if ((reinterpret_cast<uintptr_t>(scores) & 3u) || (reinterpret_cast<uintptr_t>(keep_idx) & 3u))
     return fail(ROLEKV_ERR_INVALID_ARG, "scores and keep_idx must be 4-byte aligned");
@@ -647,7 +650,7 @@ int role_alloc_select(const rolekv_batch* batch, const float* scores, const uint
   a.keep_mask = keep_mask;
   a.kept_per_role = kept_per_role;
   a.status = status_dev;
-  if (bi.n_max == 0) return ROLEKV_OK;
+  // (a batch without tokens still writes its zero per-role counts)
   stage_begin();
   cudaError_t e = launch_select(a, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "role_alloc_select");
@@ -723,17 +726,18 @@ int decode_attention(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k
   if (q.ptr == nullptr || (reinterpret_cast<uintptr_t>(q.ptr) & 15u) || q.s_head < bi.d ||
       q.s_layer < 0 || q.s_seq < 0 || (q.s_head % 8) || (q.s_seq % 8) || (q.s_layer % 8))
     return fail(ROLEKV_ERR_INVALID_ARG, "q: NULL, misaligned or bad strides");
-  if ((rc = check_tensor("k_cache", k_cache, bi.d, bi.Hkv, bi.varlen, false))) return rc;
-  if ((rc = check_tensor("v_cache", v_cache, bi.d, bi.Hkv, bi.varlen, false))) return rc;
   const int64_t bfx = to_fixed(budget);
   int64_t m_max, total;
   decode_rows(bi, batch, bfx, &m_max, &total);
+  if (total > 0) {                                 // (no rows: the outputs are zeros)
+    if ((rc = check_tensor("k_cache", k_cache, bi.d, bi.Hkv, bi.varlen, false))) return rc;
+    if ((rc = check_tensor("v_cache", v_cache, bi.d, bi.Hkv, bi.varlen, false))) return rc;
+  }
   const size_t need = decode_ws_bytes(bi, m_max);
   if (workspace == nullptr || workspace_bytes < need)
     return fail(ROLEKV_ERR_WORKSPACE, "workspace of %zu bytes, %zu needed", workspace_bytes, need);
   if (reinterpret_cast<uintptr_t>(workspace) & 255u)
     return fail(ROLEKV_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
-  if (m_max == 0) return ROLEKV_OK;
   DecodeArgs a;
   std::memset(&a, 0, sizeof(a));
   a.L = bi.L;
@@ -787,6 +791,7 @@ int kv_compact(const rolekv_batch* batch, rolekv_tensor k, rolekv_tensor v,
   if (rc) return rc;
   if (!(budget > 0.f) || budget > 1.f)
     return fail(ROLEKV_ERR_INVALID_ARG, "budget %g outside (0, 1]", static_cast<double>(budget));
+  if (bi.T == 0) return ROLEKV_OK;                 // no tokens: no kept rows
   if ((rc = check_compact_args(bi, k, v, keep_idx, k_out, v_out))) return rc;
   CompactArgs a;
   fill_compact(bi, batch->cu_seqlens_dev, to_fixed(budget), batch->seqlens_host, k, v, keep_idx,
@@ -815,6 +820,14 @@ int rolekv_compress(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tenso
   if (rc) return rc;
   SelectArgs sa;
   if ((rc = fill_select(bi, batch, params, &sa))) return rc;
+  if (bi.T == 0) {                                 // no tokens: only the zero per-role counts
+    if (kept_per_role == nullptr) return ROLEKV_OK;
+    sa.pool_k = pool_k;
+    sa.kept_per_role = kept_per_role;
+    sa.status = status_dev;
+    const cudaError_t e0 = launch_select(sa, static_cast<cudaStream_t>(stream));
+    return e0 == cudaSuccess ? ROLEKV_OK : cuda_fail(e0, "role_alloc_select");
+  }
   if (roles == nullptr || keep_idx == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "roles and keep_idx are required");
   if ((rc = check_tensor("q_win", q_win, bi.d, bi.Hq, false, true))) return rc;
   if ((rc = check_tensor("k", k, bi.d, bi.Hkv, bi.varlen, true))) return rc;

@@ -3,7 +3,8 @@ window, pool width, length mix with empty and very short sequences, budget,
 policy, recency floor), each taken through score -> select -> compact ->
 decode on the GPU and compared with the fp64 oracle: scores within 1e-3
 relative, selection and compaction bit-exact on the kernel's own scores,
-decode within the decode tolerance."""
+decode within the decode tolerance; half of them also through the H2O score
+and the Quest page bound."""
 
 import numpy as np
 import pytest
@@ -110,3 +111,44 @@ def test_random_configuration_end_to_end(seed):
                                1.0 / np.sqrt(w.d))
         got_o = o[l, s, h * w.G:(h + 1) * w.G].astype(np.float64)
         assert np.all(np.abs(got_o - r) <= 1e-3 * np.abs(r) + 1e-4 * vmax), f"seed {seed} unit {u}: decode"
+
+
+@pytest.mark.parametrize("seed", list(range(0, N_CASES, 2)))
+def test_random_configuration_h2o_and_quest(seed):
+    """The same seeded configurations through the H2O score (every causal
+    query, n kept at most 1500 for the oracle) and the Quest page bound."""
+    w, B, policy, keep_last, akey, ban = _config(seed)
+    if w.n > 1500:
+        w = w.scaled(n=1500, seqlens=None if w.seqlens is None else tuple(min(x, 1500) for x in w.seqlens))
+    roles_np = I.workload_roles(w, seed)
+    K, _ = I.make_kv(w, roles_np, seed, device=DEV, with_v=False)
+    Q = I.make_q_full(w, seed, device=DEV)
+    qw = I.make_q_window(w, seed, device=DEV)
+    batch = lib_batch(w, DEV)
+    ob = oracle_batch(w)
+    scores = torch.full(batch.score_shape(), -1.0, dtype=torch.float32, device=DEV)
+    R.h2o_score(batch, Q, K, scores)
+    torch.cuda.synchronize()
+    ref = O.h2o_batch(ob, I.bf16_bits(Q), I.bf16_bits(K))
+    got = scores.cpu().numpy()
+    for u, s in ref.items():
+        assert_scores_close(ob.score_view(got, u), s, f"seed {seed} unit {u} h2o")
+
+    page = int(np.random.default_rng(seed).choice([1, 4, 16, 33]))
+    qs = torch.full(batch.score_shape(), float("nan"), dtype=torch.float32, device=DEV)
+    R.quest_score(batch, qw, K, w.W, page, qs)
+    torch.cuda.synchronize()
+    qb, kb = I.bf16_bits(qw), I.bf16_bits(K)
+    qref = O.quest_batch(ob, qb, kb, w.W, page)
+    qgot = qs.cpu().numpy()
+    for u, r in qref.items():
+        g = ob.score_view(qgot, u).astype(np.float64)
+        l, s, h = ob.unit(u)
+        k = O.bf16_to_f64(ob.kv_rows(kb, u))
+        n = k.shape[0]
+        if n == 0:
+            continue
+        w_eff = min(w.W, n)
+        qbar = np.abs(O.bf16_to_f64(qb[l, s, h * w.G:(h + 1) * w.G, :w_eff]).reshape(-1, w.d).mean(axis=0))
+        tol = 1e-5 * qbar.sum() * np.abs(k).max() + 1e-4 * np.abs(r)
+        assert np.all(np.abs(g - r) <= tol), f"seed {seed} unit {u} quest"

@@ -184,7 +184,7 @@ struct ScorePlan {
 // chunk's tiles are still in L2 when pass 2 reads them again, large enough to
 // amortise the per-unit meeting point.  Eight chunks per unit at most: the
 // grid (152 SMs = 19 x 8) deals a unit's chunks to CTAs of the same round.
-constexpr int kFusedChunkTiles = 32;
+constexpr int kFusedChunkTiles = 64;
 constexpr int kFusedMaxChunks = 8;
 
 int64_t score_elems(const BatchInfo& bi) {

@@ -169,11 +169,6 @@ __device__ __forceinline__ int row_position(const ScoreArgs& a, int n, int rb, i
   return p < n ? p : -1;
 }
 
-__device__ __forceinline__ int num_row_blocks(const ScoreArgs& a, int n) {
-  if (a.mode == kModeSnapKV) return n > 0 ? 1 : 0;
-  return (n + a.P - 1) / a.P;
-}
-
 // Smallest position of a query block and whether every one of its rows exists.
 __device__ __forceinline__ void row_block_span(const ScoreArgs& a, int n, int rb, int* min_pos,
                                                bool* all_rows) {

@@ -160,8 +160,9 @@ def path_counts(w, B, score_kind="snapkv"):
         qbytes = U * w.G * n * d * 2
         kbytes = U * n * d * 2
         return {
-            "pass1": {"bytes": kbytes + qbytes, "flops": flops},
-            "pass2": {"bytes": kbytes + qbytes + U * n * 4, "flops": flops},
+            # one fused launch: both passes' QK^T, K and the queries read once,
+            # the scores written once
+            "score": {"bytes": kbytes + qbytes + U * n * 4, "flops": 2.0 * flops},
             "select": {"bytes": U * n * 4 + w.b * n + U * K * 4, "flops": 0.0},
             "compact": {"bytes": U * K * 4 + 2 * 2 * U * K * d * 2, "flops": 0.0},
             "path_bytes": kbytes + qbytes + U * n * 8 + U * K * 8 + 2 * 2 * U * K * d * 2 + w.b * n,
@@ -222,7 +223,7 @@ def run_gpu(args):
     status = torch.zeros(1, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream(dev)
 
-    names = ["pass1", "pass2", "select", "compact"] if h2o else ["score", "select", "compact"]
+    names = ["score", "select", "compact"]
     # the Quest page bound is selected as it is (no max-pool over the KV axis)
     pool_k = 1 if args.score == "quest" else w.pool_k
     ns = len(names) - 2                              # score kernels

@@ -18,6 +18,12 @@
 // tcgen05.mma (bf16 operands, fp32 accumulators in tensor memory, two
 // accumulator buffers) and sixteen epilogue warps drain the accumulators with
 // tcgen05.ld.  Every wait is an mbarrier wait bounded in time.
+//
+// snapkv_fused_kernel runs both passes in one persistent launch, for SnapKV
+// (items = chunks of a unit's keys; the chunks of a unit exchange their row
+// statistics through global memory between the passes) and for H2O (items =
+// query blocks; a block's normalisers are its own, so they stay on chip).
+// attn_pass_kernel runs one pass per launch (the no-workspace SnapKV call).
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -713,7 +719,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// ------------------------------------------------------------ fused SnapKV --
+// ------------------------------------------------- fused SnapKV / H2O score --
 
 template <int D>
 struct FCfg {
@@ -803,6 +809,35 @@ __device__ __forceinline__ void chunk_tiles(const ScoreArgs& a, int n, int c, in
   const int ct = (ntiles + a.n_chunks - 1) / a.n_chunks;
   *kt0 = min(ntiles, c * ct);
   *kt1 = min(ntiles, *kt0 + ct);
+}
+
+// Item `item` of the fused launch.  SnapKV: (unit, chunk of its key tiles).
+// H2O: (unit, query block), the longest blocks first, over the key tiles up
+// to the block's last position; its rows' normalisers are its own (no other
+// CTA contributes), so the block needs no cross-CTA exchange.
+struct FItem {
+  int u, chunk, rb, kt0, kt1;
+  Unit un;
+};
+
+__device__ __forceinline__ FItem fused_item(const ScoreArgs& a, int item) {
+  FItem it;
+  if (a.mode == kModeSnapKV) {
+    it.u = item / a.n_chunks;
+    it.chunk = item % a.n_chunks;
+    it.rb = 0;
+    it.un = decode_unit(a, it.u);
+    chunk_tiles(a, it.un.n, it.chunk, &it.kt0, &it.kt1);
+  } else {
+    it.u = item % a.n_units;
+    it.chunk = 0;
+    it.rb = a.nrb_max - 1 - item / a.n_units;
+    it.un = decode_unit(a, it.u);
+    const int n = it.un.n;
+    it.kt0 = 0;
+    it.kt1 = (it.rb * a.P < n) ? (min(n, (it.rb + 1) * a.P) + kTileKeys - 1) / kTileKeys : 0;
+  }
+  return it;
 }
 
 template <int D>
@@ -900,17 +935,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       int kload = 0, qload = 0;
       // Items are dealt round-robin: the grid is a multiple of the chunks per
       // unit, so a unit's chunks run on different CTAs in the same round.
+      const bool h2o = a.mode == kModeH2O;
       for (int item = blockIdx.x; item < fa.n_items; item += gridDim.x) {
-        const Unit un = decode_unit(a, item / a.n_chunks);
-        int kt0, kt1;
-        chunk_tiles(a, un.n, item % a.n_chunks, &kt0, &kt1);
+        const FItem it = fused_item(a, item);
+        const Unit& un = it.un;
+        const int kt0 = it.kt0, kt1 = it.kt1;
         if (kt1 == kt0) continue;
-        // window queries of the unit
+        // the item's query rows: the unit's window (SnapKV) or query block (H2O)
         if (!mbar_wait(sh.q_empty, (qload & 1) ^ 1, sh.abort_flag, a.status)) break;
         mbar_arrive_expect_tx(sh.q_full, static_cast<uint32_t>(a.nrows) * D * 2);
         for (int g = 0; g < a.G; ++g) {
-          const Coord c = tma_coord(a.q_layer, a.q_seq, a.q_head, a.q_tok, false, un,
-                                    un.h * a.G + g, 0);
+          const Coord c = tma_coord(a.q_layer, a.q_seq, a.q_head, a.q_tok, h2o && a.varlen != 0, un,
+                                    un.h * a.G + g, h2o ? static_cast<int64_t>(it.rb) * a.P : 0);
 #pragma unroll
           for (int hf = 0; hf < C::kHalves; ++hf)
             tma_load_2d_hint(sh.q + hf * C::kQHalfBytes + g * a.P * 128, &q_map, c.x + hf * 64,
@@ -952,9 +988,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       int kuse = 0, quse = 0, pair = 0;
       bool ok = true;
       for (int item = blockIdx.x; item < fa.n_items && ok; item += gridDim.x) {
-        const Unit un = decode_unit(a, item / a.n_chunks);
-        int kt0, kt1;
-        chunk_tiles(a, un.n, item % a.n_chunks, &kt0, &kt1);
+        const FItem it = fused_item(a, item);
+        const int kt0 = it.kt0, kt1 = it.kt1;
         if (kt1 == kt0) continue;
         if (!mbar_wait(sh.q_full, quse & 1, sh.abort_flag, a.status)) break;
         ++quse;
@@ -1015,17 +1050,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     int pair = 0, xchg = 0;
     bool ok = true;
     int ipop = 0;                                  // items done: barrier phases
-    for (int item = blockIdx.x; item < fa.n_items && ok; item += gridDim.x, ++ipop) {
-      const int u = item / a.n_chunks;
-      const int chunk = item % a.n_chunks;
-      const Unit un = decode_unit(a, u);
+    const bool h2o = a.mode == kModeH2O;
+    for (int item = blockIdx.x; item < fa.n_items && ok; item += gridDim.x) {
+      const FItem it = fused_item(a, item);
+      const int u = it.u, chunk = it.chunk, rb = it.rb;
+      const Unit& un = it.un;
       const int n = un.n;
-      int kt0, kt1;
-      chunk_tiles(a, n, chunk, &kt0, &kt1);
+      const int kt0 = it.kt0, kt1 = it.kt1;
+      if (h2o && kt1 == kt0) continue;           // a block past its sequence's end
 
       if (!fa.single) {
       // ---- pass 1: running (max2, sum) of this thread's row over its keys
-      const int pos = row_position(a, n, 0, row);
+      const int pos = row_position(a, n, rb, row);
       float m2 = -INFINITY, l = 0.f;
       for (int kt = kt0; kt < kt1; ++kt, ++pair) {
         const int ab = pair & 1;
@@ -1058,10 +1094,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             m2 = mm;
           }
         }
-        const int64_t slot = static_cast<int64_t>(u) * a.n_chunks + chunk;
-        a.partials[slot * kRowsMax + row] = make_float2(m2, l);
-        if (nrt == 1) a.partials[slot * kRowsMax + 128 + row] = make_float2(-INFINITY, 0.f);
-        __threadfence();
+        if (h2o) {
+          sh.merge[row] = make_float2(m2, l);      // (slot 0: the leader's own)
+        } else {
+          const int64_t slot = static_cast<int64_t>(u) * a.n_chunks + chunk;
+          a.partials[slot * kRowsMax + row] = make_float2(m2, l);
+          if (nrt == 1) a.partials[slot * kRowsMax + 128 + row] = make_float2(-INFINITY, 0.f);
+          __threadfence();
+        }
       }
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) break;
@@ -1070,7 +1110,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // every row of this chunk is visible: count it, then wait for the
         // unit's other chunks (bounded)
         bool got = mbar_wait(sh.pub, ipop & 1, sh.abort_flag, a.status);
-        if (got) {
+        if (got && !h2o) {
           __threadfence();
           atomicAdd(fa.work + 1 + u, 1);
           const uint64_t t0 = global_timer_ns();
@@ -1093,9 +1133,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       // with caller-supplied window normalisers, as snapkv_lse_kernel wrote them)
       if (etid < kRowsMax) {
         const int j = etid;
-        const int p = row_position(a, n, 0, j);
+        const int p = row_position(a, n, rb, j);
         float nl = -INFINITY;
-        if (fa.single) {
+        if (h2o) {
+          const float2 ml = sh.merge[j];
+          if (p >= 0 && ml.y > 0.f) nl = -(ml.x + log2f(ml.y));
+        } else if (fa.single) {
           nl = (p >= 0) ? a.lse2[static_cast<int64_t>(u) * kRowsMax + j] : -INFINITY;
         } else if (p >= 0) {
           // one online merge over the chunks, eight independent loads in flight
@@ -1128,7 +1171,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // ---- pass 2: column sums of this thread's key over its rows
       int min_pos;
       bool all_rows;
-      row_block_span(a, n, 0, &min_pos, &all_rows);
+      row_block_span(a, n, rb, &min_pos, &all_rows);
       const int64_t sbase = score_base(a, un, u);
       for (int kt = kt0; kt < kt1; ++kt, ++pair) {
         const int t = kt * kTileKeys + kl;
@@ -1183,10 +1226,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!ok) break;
           const float total = colsum + sh.red[grp * kTileKeys + kl];
           mbar_arrive(&sh.red_empty[grp]);
-          if (t < n) a.prepool[sbase + t] = total;
+          if (t < n) {
+            if (h2o)
+              atomicAdd(a.prepool + sbase + t, total);   // one query block's share
+            else
+              a.prepool[sbase + t] = total;
+          }
         }
         ++xchg;
       }
+      ++ipop;
     }
   }
 

@@ -195,7 +195,7 @@ int plan_score(int mode, const BatchInfo& bi, int W, bool need_partials, bool ne
                ScorePlan* p, bool fused = false) {
   ScoreArgs& a = p->a;
   std::memset(&a, 0, sizeof(a));
-  p->fused = fused && mode == kModeSnapKV;
+  p->fused = fused;
   if (bi.d != 64 && bi.d != 128)
     return fail(ROLEKV_ERR_UNSUPPORTED, "head dim %d (the score kernels take 64 or 128)", bi.d);
   a.L = bi.L;
@@ -240,12 +240,15 @@ int plan_score(int mode, const BatchInfo& bi, int W, bool need_partials, bool ne
     a.nrb_max = (bi.n_max + a.P - 1) / a.P;
     p->grid1 = a.n_units * a.nrb_max;
     p->grid2 = p->grid1;                          // pass 2 per query block too
+    a.n_chunks = 1;                               // (fused: no cross-CTA exchange)
+    p->n_items = a.n_units * a.nrb_max;
   }
   size_t off = 256;   // first 256 bytes reserved
   p->off_partials = off;
   if (need_partials) off += align256(static_cast<size_t>(a.n_units) * a.n_chunks * kRowsMax * 8);
   p->off_lse = off;
-  off += align256(static_cast<size_t>(a.n_units) * a.nrb_max * kRowsMax * 4);
+  if (!(p->fused && mode == kModeH2O))           // the fused H2O keeps its normalisers on chip
+    off += align256(static_cast<size_t>(a.n_units) * a.nrb_max * kRowsMax * 4);
   p->off_prepool = off;
   if (need_prepool) off += align256(static_cast<size_t>(score_elems(bi)) * 4);
   p->off_work = off;
@@ -496,7 +499,7 @@ int rolekv_workspace_size(int op, const rolekv_batch* batch, int32_t W, size_t* 
   ScorePlan p;
   switch (op) {
     case 0: rc = plan_score(kModeSnapKV, bi, W, true, true, &p, true); break;
-    case 1: rc = plan_score(kModeH2O, bi, 0, false, false, &p); break;
+    case 1: rc = plan_score(kModeH2O, bi, 0, false, false, &p, true); break;
     case 2: rc = plan_score(kModeSnapKV, bi, W, true, true, &p, true); break;
     default: return fail(ROLEKV_ERR_INVALID_ARG, "unknown op %d", op);
   }
@@ -546,7 +549,7 @@ int h2o_score(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k, float
   int rc = check_batch(batch, &bi);
   if (rc) return rc;
   ScorePlan p;
-  rc = plan_score(kModeH2O, bi, 0, false, false, &p);
+  rc = plan_score(kModeH2O, bi, 0, false, false, &p, true);
   if (rc) return rc;
   if (bi.T == 0) return ROLEKV_OK;                 // no tokens: nothing to score
   if (scores == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "scores is NULL");
@@ -568,14 +571,18 @@ int h2o_score(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k, float
   if (rc) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   stage_begin();
-  cudaError_t e = launch_attn_pass(0, bi.d, kmap, qmap, a, p.grid1, st);
-  if (e != cudaSuccess) return cuda_fail(e, "h2o pass 1");
-  // pass 2 adds every query block's column sums into the scores
-  e = cudaMemsetAsync(scores, 0, static_cast<size_t>(score_elems(bi)) * sizeof(float), st);
+  // every query block adds its column sums into the zeroed scores
+  cudaError_t e = cudaMemsetAsync(scores, 0, static_cast<size_t>(score_elems(bi)) * sizeof(float), st);
   if (e != cudaSuccess) return cuda_fail(e, "clearing the scores");
-  stage_mark(st);
-  e = launch_attn_pass(1, bi.d, kmap, qmap, a, p.grid2, st);
-  if (e != cudaSuccess) return cuda_fail(e, "h2o pass 2");
+  // one persistent launch: per query block, its row normalisers (pass 1)
+  // then its share of the column sums (pass 2)
+  FusedArgs fa;
+  fa.s = a;
+  fa.work = p.work;
+  fa.n_items = p.n_items;
+  fa.single = 0;
+  e = launch_snapkv_fused(bi.d, kmap, qmap, fa, st);
+  if (e != cudaSuccess) return cuda_fail(e, "h2o fused score");
   stage_mark(st);
   return ROLEKV_OK;
 }

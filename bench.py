@@ -482,11 +482,16 @@ def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_o
             stream, world, seq_tokens):
     """The same step through the public calls with host buffers: the step's
     inputs are copied from pinned host memory and the kept indices and the
-    compressed K/V read back, inside the timed region."""
+    compressed K/V read back, inside the timed region.  The step runs layer
+    slice by layer slice on three streams, so that a slice's host-to-device
+    copy, another slice's kernels and a third slice's read-back overlap (as
+    a prefill that hands its cache over layer by layer would)."""
     import torch
 
     from paper_2607_13205_gb300 import rolekv as R
 
+    h2o = w.kind == "h2o"
+    dev = K.device
     h_qw = torch.empty(qw.shape, dtype=qw.dtype, pin_memory=True)
     h_k = torch.empty(K.shape, dtype=K.dtype, pin_memory=True)
     h_v = torch.empty(V.shape, dtype=V.dtype, pin_memory=True)
@@ -502,18 +507,62 @@ def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_o
     bi = sum(t.numel() * t.element_size() for t in (h_qw, h_k, h_v, h_roles))
     bo = sum(t.numel() * t.element_size() for t in (o_keep, o_k, o_v))
 
-    def e2e_step():
-        qw.copy_(h_qw, non_blocking=True)
-        K.copy_(h_k, non_blocking=True)
-        V.copy_(h_v, non_blocking=True)
-        roles.copy_(h_roles, non_blocking=True)
-        score()
-        R.role_alloc_select(batch, scores, roles, params, keep, pool_k=(1 if args.score == "quest" else w.pool_k), status=status,
+    # layer slices; every tensor of the path has the layer axis first
+    S = min(w.L, 8)
+    bounds = [(w.L * i // S, w.L * (i + 1) // S) for i in range(S)]
+    seqlens = list(w.seqlens) if w.varlen else None
+    sbatch = {}
+    for l0, l1 in bounds:
+        if l1 - l0 not in sbatch:
+            sbatch[l1 - l0] = R.Batch(l1 - l0, w.b, w.Hq, w.Hkv, w.d, w.n, seqlens=seqlens, device=dev)
+    big = sbatch[max(sbatch)]
+    ws = R.workspace(R.OP_H2O if h2o else R.OP_SNAPKV, big, w.W, device=dev)
+    pool_k = 1 if args.score == "quest" else w.pool_k
+    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    ev_roles = torch.cuda.Event()
+    ev_in = [torch.cuda.Event() for _ in bounds]
+    ev_done = [torch.cuda.Event() for _ in bounds]
+    ev_out = [torch.cuda.Event() for _ in bounds]
+
+    def slice_kernels(i):
+        l0, l1 = bounds[i]
+        sb = sbatch[l1 - l0]
+        if h2o:
+            R.h2o_score(sb, qw[l0:l1], K[l0:l1], scores[l0:l1], ws=ws, status=status, stream=stream)
+        elif args.score == "quest":
+            R.quest_score(sb, qw[l0:l1], K[l0:l1], w.W, args.page, scores[l0:l1], stream=stream)
+        else:
+            R.snapkv_score(sb, qw[l0:l1], K[l0:l1], w.W, 1, scores[l0:l1], ws=ws, status=status,
+                           stream=stream)
+        R.role_alloc_select(sb, scores[l0:l1], roles, params, keep[l0:l1], pool_k=pool_k, status=status,
                             stream=stream)
-        R.kv_compact(batch, K, V, keep, B, k_out, v_out, status=status, stream=stream)
-        o_keep.copy_(keep, non_blocking=True)
-        o_k.copy_(k_out, non_blocking=True)
-        o_v.copy_(v_out, non_blocking=True)
+        R.kv_compact(sb, K[l0:l1], V[l0:l1], keep[l0:l1], B, k_out[l0:l1], v_out[l0:l1], status=status,
+                     stream=stream)
+
+    def e2e_step():
+        with torch.cuda.stream(s_in):
+            s_in.wait_event(ev_done[-1])              # the roles' last use by the kernels
+            roles.copy_(h_roles, non_blocking=True)
+            ev_roles.record(s_in)
+            for i, (l0, l1) in enumerate(bounds):
+                s_in.wait_event(ev_done[i])            # the slice's last use by the kernels
+                qw[l0:l1].copy_(h_qw[l0:l1], non_blocking=True)
+                K[l0:l1].copy_(h_k[l0:l1], non_blocking=True)
+                V[l0:l1].copy_(h_v[l0:l1], non_blocking=True)
+                ev_in[i].record(s_in)
+        stream.wait_event(ev_roles)
+        for i in range(S):
+            stream.wait_event(ev_in[i])
+            stream.wait_event(ev_out[i])               # the slice's outputs were read back
+            slice_kernels(i)
+            ev_done[i].record(stream)
+        with torch.cuda.stream(s_out):
+            for i, (l0, l1) in enumerate(bounds):
+                s_out.wait_event(ev_done[i])
+                o_keep[l0:l1].copy_(keep[l0:l1], non_blocking=True)
+                o_k[l0:l1].copy_(k_out[l0:l1], non_blocking=True)
+                o_v[l0:l1].copy_(v_out[l0:l1], non_blocking=True)
+                ev_out[i].record(s_out)
 
     e2e_step()
     torch.cuda.synchronize()
@@ -528,7 +577,8 @@ def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_o
     barrier(world)
     dt = max_over_ranks(dt, world)
     return {"value": world * seq_tokens * steps / dt, "unit": UNIT, "h2d_bytes_per_step": bi,
-            "d2h_bytes_per_step": bo, "steps": steps, "ms_per_step": dt / steps * 1e3}
+            "d2h_bytes_per_step": bo, "steps": steps, "ms_per_step": dt / steps * 1e3,
+            "slices": S, "overlap": "layer slices: copy in, kernels and read-back on three streams"}
 
 
 # ------------------------------------------------------ CPU oracle baseline --

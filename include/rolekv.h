@@ -247,7 +247,9 @@ int decode_attention(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k
  * of the KV head and every causal query position q >= t of p_t(q).
  *   q       bf16 prefill queries of every position: dense [L][b][Hq][n][d] or
  *           varlen [L][T][Hq][d], addressed by its strides.
- *   scores  fp32 score array.  No pooling (the H2O score has none).
+ *   scores  fp32 score array.  No pooling (the H2O score has none).  Each
+ *           score is a sum of per-query-block parts added atomically, in an
+ *           order that varies between runs (about 1e-7 relative).
  * d must be 64 or 128 and G <= 8. */
 int h2o_score(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k, float scale,
               float* scores, void* workspace, size_t workspace_bytes, int32_t* status_dev,

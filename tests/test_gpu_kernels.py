@@ -606,3 +606,37 @@ def test_bounded_wait_reports_timeout():
     assert 0.015 <= dt < 5.0
     x = torch.arange(8, device=DEV).sum()        # the context still works
     assert int(x.item()) == 28
+
+
+@pytest.mark.parametrize("varlen", [False, True])
+def test_layer_slices_match_whole_batch(varlen):
+    """The calls on layer slices of the tensors (views with a storage offset,
+    a batch of fewer layers) give exactly the whole batch's scores, kept
+    indices and compressed rows, as a prefill handing over its cache layer by
+    layer would use them."""
+    w = (_w("ragged", L=4, b=3, Hq=8, Hkv=2, n=2000, seqlens=(2000, 700, 0)) if varlen
+         else _w("llama8b", L=4, b=2, Hq=8, Hkv=2, n=2500))
+    roles_np, K, V, qw = _snapkv_inputs(w, seed=11)
+    roles = torch.as_tensor(roles_np, device=DEV)
+    B = 0.1
+    params = R.select_params(B, I.PAPER_ALPHA, 0.02, I.ROLE_KEY)
+    full = lib_batch(w, DEV)
+
+    def run(batch, q, k, v):
+        sc = torch.empty(batch.score_shape(), dtype=torch.float32, device=DEV)
+        R.snapkv_score(batch, q, k, w.W, 1, sc)
+        kp = torch.empty(batch.kept_shape(B), dtype=torch.int32, device=DEV)
+        R.role_alloc_select(batch, sc, roles, params, kp, pool_k=w.pool_k)
+        ko = torch.empty(R.compact_shape(batch, B), dtype=torch.bfloat16, device=DEV)
+        vo = torch.empty_like(ko)
+        R.kv_compact(batch, k, v, kp, B, ko, vo)
+        return sc, kp, ko, vo
+
+    whole = run(full, qw, K, V)
+    half = _w(w.name, **{f: getattr(w, f) for f in ("b", "Hq", "Hkv", "d", "n", "W", "pool_k", "seqlens")},
+              L=2)
+    sb = lib_batch(half, DEV)
+    parts = [run(sb, qw[l0:l0 + 2], K[l0:l0 + 2], V[l0:l0 + 2]) for l0 in (0, 2)]
+    torch.cuda.synchronize()
+    for x, (a, b) in enumerate(zip(whole, zip(*parts))):
+        assert torch.equal(torch.cat(b, dim=0), a), f"output {x}"

@@ -29,12 +29,14 @@ matmul / sort as the only library steps:
                            top-ceil(alpha_r B n_kv) per role bucket, alpha
                            renormalised over buckets, slack from saturated
                            buckets redistributed (Section 4.1; Algorithm 1).
-                           Three more splits: GLOBAL (plain top-k, optional
+                           Four more splits: GLOBAL (plain top-k, optional
                            role ban; Sections 2 and 4), FAIR (equal
                            retention rate per role; Section 5
-                           "Fair-eviction baseline") and SLACK (the slack of
+                           "Fair-eviction baseline"), SLACK (the slack of
                            saturated buckets filled by score instead of
-                           in proportion to alpha).
+                           in proportion to alpha) and CEIL (Algorithm 1's
+                           per-bucket ceilings taken literally, so the
+                           total may exceed ceil(B n)).
 * ``select_unit``       -- per-bucket top-q_r by pooled score (Algorithm 1);
                            ``select_batch`` optionally keeps the last R
                            tokens first (SnapKV's recency floor, Section 7).
@@ -68,6 +70,7 @@ POLICY_ROLE_QUOTA = 0
 POLICY_GLOBAL = 1
 POLICY_FAIR = 2
 POLICY_SLACK = 3
+POLICY_CEIL = 4
 
 
 # ----------------------------------------------------------------------------
@@ -264,6 +267,14 @@ def role_quotas(counts: Sequence[int], alpha: Sequence[float], budget: float, n:
     fills that slack with the best-scoring remaining tokens of the eligible
     buckets.
 
+    CEIL (Algorithm 1 read literally: bucket r keeps the top
+    ceil(alpha_r B n_kv) of its tokens, alpha renormalised over the eligible
+    buckets): the ROLE_QUOTA water-filling of saturated buckets, then every
+    unsaturated bucket takes the ceiling of its share instead of floor plus
+    largest remainder.  Each ceiling exceeds its share by less than one, so
+    the quotas sum to between K and K + (unsaturated buckets - 1); the rows
+    that hold them must be that much wider than ceil(B n) (Batch.kept_extra).
+
     k_full, when given, replaces ceil(B n) as the budget to split (the
     recency floor of select_batch takes its tokens out of it first).
     """
@@ -294,7 +305,11 @@ def role_quotas(counts: Sequence[int], alpha: Sequence[float], budget: float, n:
             q[r] = counts[r]
             k_left -= counts[r]
         S = [r for r in S if r not in saturated]
-    if S:
+    if S and policy == POLICY_CEIL:
+        A = sum(a[r] for r in S)
+        for r in S:
+            q[r] = -((-a[r] * k_left) // A)          # ceil(a_r k_left / A)
+    elif S:
         A = sum(a[r] for r in S)
         rem = {}
         for r in S:
@@ -367,8 +382,9 @@ class Batch:
     [L][b][Hq][W][d]."""
 
     def __init__(self, L: int, b: int, Hq: int, Hkv: int, d: int, n_max: int,
-                 seqlens: Iterable[int] | None = None):
+                 seqlens: Iterable[int] | None = None, kept_extra: int = 0):
         self.L, self.b, self.Hq, self.Hkv, self.d, self.n_max = L, b, Hq, Hkv, d, n_max
+        self.kept_extra = int(kept_extra)
         if Hq % Hkv:
             raise ValueError("Hq must be a multiple of Hkv")
         self.G = Hq // Hkv
@@ -415,8 +431,13 @@ class Batch:
             return scores[l, h, self.cu[s]:self.cu[s] + n]
         return scores[l, s, h, :n]
 
+    def kept_rows(self, n: int, budget: float) -> int:
+        """Width of an n-token sequence's kept row: ceil(B n) slots plus
+        kept_extra (room for the CEIL split's overshoot), at most n."""
+        return min(n, kept_count(n, budget) + self.kept_extra) if n > 0 else 0
+
     def kept_offsets(self, budget: float) -> np.ndarray:
-        ks = [kept_count(n, budget) if n > 0 else 0 for n in self.seqlens]
+        ks = [self.kept_rows(n, budget) for n in self.seqlens]
         return np.concatenate([[0], np.cumsum(ks)]).astype(np.int64)
 
 
@@ -469,8 +490,8 @@ def select_batch(batch: Batch, unit_scores: dict, roles, n_roles: int, alpha: Se
     R = min(keep_last, n, ceil(B n)) tokens are kept whatever their score and
     role, and the remaining ceil(B n) - R slots are split over the earlier
     tokens exactly as without the floor (roles counted over those tokens
-    only).  Returns {unit: (kept_idx padded with -1 to ceil(B n), kept count
-    per role)}.
+    only).  Returns {unit: (kept_idx padded with -1 to the row width
+    batch.kept_rows(n, B), kept count per role)}.
     """
     al = [float(np.float32(a)) for a in alpha[:n_roles]]
     if 0 <= key_role < n_roles:
@@ -480,11 +501,12 @@ def select_batch(batch: Batch, unit_scores: dict, roles, n_roles: int, alpha: Se
         _, s, _ = batch.unit(u)
         r = np.asarray(batch.roles(roles, s)).astype(np.int64)
         n = r.shape[0]
-        width = kept_count(n, budget) if n > 0 else 0
-        forced = min(int(keep_last), n, width)
+        budget_n = kept_count(n, budget) if n > 0 else 0
+        width = batch.kept_rows(n, budget)
+        forced = min(int(keep_last), n, budget_n)
         nf = n - forced                              # tokens before the floor
         counts = [int((r[:nf] == x).sum()) for x in range(n_roles)]
-        q = role_quotas(counts, al, budget, n, policy, ban_mask, k_full=width - forced)
+        q = role_quotas(counts, al, budget, n, policy, ban_mask, k_full=budget_n - forced)
         bk = bucket_of_tokens(r, policy, ban_mask)
         bk[nf:] = -1
         idx = select_unit(np.asarray(sc, dtype=np.float64), bk, q)
@@ -492,7 +514,7 @@ def select_batch(batch: Batch, unit_scores: dict, roles, n_roles: int, alpha: Se
             # the slack of saturated buckets goes to the best-scoring tokens
             # of eligible buckets not kept yet (ties to the lower index)
             E = eligible_roles(counts, al, policy, ban_mask)
-            K = min(width - forced, sum(counts[x] for x in E))
+            K = min(budget_n - forced, sum(counts[x] for x in E))
             slack = K - sum(q)
             if slack > 0:
                 sc64 = np.asarray(sc, dtype=np.float64)

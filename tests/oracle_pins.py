@@ -448,6 +448,56 @@ def pin_slack_fill(O, rng):
             assert per[2] == 0
 
 
+def pin_ceil_quotas(O, rng):
+    """CEIL (Algorithm 1's per-bucket ceilings read literally): hand-worked
+    quotas; every eligible bucket takes the ceiling of its exact water-level
+    share (an independent formulation), so no quota is below the exact
+    split's, the total exceeds K by less than the number of unsaturated
+    buckets, and the kept set contains the exact split's; rows are padded
+    with -1 to min(n, ceil(B n) + kept_extra)."""
+    for ex in _golden("ceil_quota_worked_examples.json")["examples"]:
+        q = O.role_quotas(ex["counts"], ex["alpha"], ex["budget"], ex["n"], policy=O.POLICY_CEIL)
+        assert q == ex["quotas"], (ex["name"], q, ex["quotas"])
+        assert sum(q) == ex["kept"]
+    for _ in range(400):
+        R = int(rng.integers(1, 9))
+        counts = [int(x) for x in rng.integers(0, 60, size=R)]
+        n = sum(counts)
+        if n == 0:
+            continue
+        alpha = [float(np.float32(x)) for x in rng.choice([0.0, 0.02, 0.05, 0.2, 0.25, 0.7, 0.33], size=R)]
+        B = float(rng.choice([0.05, 0.1, 0.2, 0.3, 0.5, 0.9, 1.0]))
+        q = O.role_quotas(counts, alpha, B, n, policy=O.POLICY_CEIL)
+        q0 = O.role_quotas(counts, alpha, B, n)
+        w = [round(a * 1e6) for a in alpha]
+        elig = sum(c for c, a in zip(counts, w) if a > 0)
+        K = min(math.ceil(Fraction(round(B * 1e6), 10**6) * n), elig)
+        ideal = _water_level(counts, w, K)
+        for r in range(R):
+            assert q[r] == (math.ceil(ideal[r]) if r in ideal else 0), (counts, alpha, B, q, r)
+            assert q0[r] <= q[r] <= counts[r]
+        unsat = sum(1 for r in ideal if ideal[r] < counts[r])
+        assert K <= sum(q) <= K + max(unsat - 1, 0), (counts, alpha, B, q, K)
+    b, n = 2, 500
+    for extra in (3, 7):
+        batch = O.Batch(1, b, 2, 1, 8, n, kept_extra=extra)
+        roles = rng.integers(0, 4, size=(b, n)).astype(np.uint8)
+        sc = {u: rng.random(n) for u in range(b)}
+        al = [0.25, 0.02, 0.70, 0.05]
+        for B, keep_last in ((0.05, 0), (0.13, 0), (0.3, 16), (0.999, 0)):
+            ceil_sel = O.select_batch(batch, sc, roles, 4, al, -1, 0.0, B, O.POLICY_CEIL, keep_last=keep_last)
+            exact_sel = O.select_batch(batch, sc, roles, 4, al, -1, 0.0, B, keep_last=keep_last)
+            width = min(n, math.ceil(Fraction(round(B * 1e6), 10**6) * n) + extra)
+            for u in range(b):
+                idx, per = ceil_sel[u]
+                assert idx.shape == (width,)
+                kept = idx[idx >= 0]
+                assert np.all(idx[kept.size:] == -1) and np.all(np.diff(kept) > 0)
+                assert set(exact_sel[u][0][exact_sel[u][0] >= 0]) <= set(kept)
+                assert sum(per) == kept.size
+                assert np.all(kept[kept.size - keep_last:] == np.arange(n - keep_last, n)) if keep_last else True
+
+
 def pin_recency_floor(O, rng):
     """The recency floor keeps the last R = min(keep_last, n, ceil(B n))
     tokens and splits the other ceil(B n) - R slots over the earlier tokens:
@@ -553,4 +603,5 @@ ALL_PINS = [
     pin_kept_count, pin_quota_golden, pin_quota_waterlevel, pin_key_ban,
     pin_global_is_full_sort, pin_bruteforce_select, pin_compact, pin_varlen_matches_dense,
     pin_fair_quotas, pin_recency_floor, pin_quest_bound, pin_decode_attention, pin_slack_fill,
+    pin_ceil_quotas,
 ]

@@ -190,7 +190,7 @@ def _m_fair_uses_alpha(O):
 
 
 def _m_floor_outside_budget(O):
-    _from_source(O, "k_full=width - forced)", "k_full=width)", ["select_batch"])
+    _from_source(O, "k_full=budget_n - forced)", "k_full=budget_n)", ["select_batch"])
 
 
 def _m_floor_counts_whole_row(O):
@@ -227,6 +227,23 @@ def _m_slack_not_filled(O):
     _from_source(O, "if slack > 0:", "if slack > 10**9:", ["select_batch"])
 
 
+def _m_ceil_floors(O):
+    _from_source(O, "q[r] = -((-a[r] * k_left) // A)", "q[r] = (a[r] * k_left) // A", ["role_quotas"])
+
+
+def _m_ceil_no_waterfill(O):
+    _from_source(O, "while S and policy != POLICY_SLACK:", "while S and policy not in (POLICY_SLACK, POLICY_CEIL):",
+                 ["role_quotas"])
+
+
+def _m_ceil_unnormalised(O):
+    _from_source(O, "q[r] = -((-a[r] * k_left) // A)", "q[r] = -((-a[r] * k_left) // FIXED_ONE)", ["role_quotas"])
+
+
+def _m_ceil_rows_not_widened(O):
+    _from_source(O, "width = batch.kept_rows(n, budget)", "width = budget_n", ["select_batch"])
+
+
 def _m_compact_off_by_one(O):
     orig = O.compact_unit
     O.compact_unit = lambda rows, idx: orig(rows, np.where(np.asarray(idx) >= 0, np.minimum(np.asarray(idx) + 1, rows.shape[0] - 1), -1))
@@ -239,7 +256,8 @@ MUTATIONS = [
     _m_ties_to_high_index, _m_interleaved_gqa, _m_compact_off_by_one, _m_fair_uses_alpha,
     _m_floor_outside_budget, _m_floor_counts_whole_row, _m_quest_max_only, _m_quest_window_start,
     _m_decode_keeps_padding, _m_decode_unnormalised, _m_slack_from_all_roles, _m_slack_waterfills,
-    _m_slack_not_filled,
+    _m_slack_not_filled, _m_ceil_floors, _m_ceil_no_waterfill, _m_ceil_unnormalised,
+    _m_ceil_rows_not_widened,
 ]
 
 

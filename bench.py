@@ -210,9 +210,8 @@ def run_gpu(args):
     qw = I.make_q_full(w, seed=rank, device=dev) if h2o else I.make_q_window(w, seed=rank, device=dev)
     roles = torch.as_tensor(roles_np, device=dev)
     batch = R.Batch(w.L, w.b, w.Hq, w.Hkv, w.d, w.n, seqlens=list(w.seqlens) if w.varlen else None,
-                    device=dev)
-    policy = {"quota": R.POLICY_ROLE_QUOTA, "global": R.POLICY_GLOBAL, "fair": R.POLICY_FAIR,
-              "slack": R.POLICY_SLACK}[args.policy]
+                    device=dev, kept_extra=kept_extra(args.policy))
+    policy = POLICY_CODES[args.policy]
     params = R.select_params(B, I.PAPER_ALPHA, alpha_key=0.0, key_role=I.ROLE_KEY, policy=policy,
                              keep_last=args.keep_last)
     scores = torch.empty(batch.score_shape(), dtype=torch.float32, device=dev)
@@ -514,7 +513,8 @@ def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_o
     sbatch = {}
     for l0, l1 in bounds:
         if l1 - l0 not in sbatch:
-            sbatch[l1 - l0] = R.Batch(l1 - l0, w.b, w.Hq, w.Hkv, w.d, w.n, seqlens=seqlens, device=dev)
+            sbatch[l1 - l0] = R.Batch(l1 - l0, w.b, w.Hq, w.Hkv, w.d, w.n, seqlens=seqlens, device=dev,
+                                      kept_extra=kept_extra(args.policy))
     big = sbatch[max(sbatch)]
     ws = R.workspace(R.OP_H2O if h2o else R.OP_SNAPKV, big, w.W, device=dev)
     pool_k = 1 if args.score == "quest" else w.pool_k
@@ -583,7 +583,13 @@ def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_o
 
 # ------------------------------------------------------ CPU oracle baseline --
 
-POLICY_CODES = {"quota": 0, "global": 1, "fair": 2, "slack": 3}
+POLICY_CODES = {"quota": 0, "global": 1, "fair": 2, "slack": 3, "ceil": 4}
+
+
+def kept_extra(policy: str) -> int:
+    """Kept-row slots beyond ceil(B n): the ceiling split's total can exceed
+    the budget by one slot per weighted role but one."""
+    return 3 if policy == "ceil" else 0      # four roles
 
 
 def oracle_units(w, B, units, qw_bits, k_bits, v_bits, roles_np, policy="quota", keep_last=0,
@@ -592,7 +598,8 @@ def oracle_units(w, B, units, qw_bits, k_bits, v_bits, roles_np, policy="quota",
     from oracle import rolekv_oracle as O
     from paper_2607_13205_gb300 import inputs as I
 
-    ob = O.Batch(w.L, w.b, w.Hq, w.Hkv, w.d, w.n, seqlens=list(w.seqlens) if w.varlen else None)
+    ob = O.Batch(w.L, w.b, w.Hq, w.Hkv, w.d, w.n, seqlens=list(w.seqlens) if w.varlen else None,
+                 kept_extra=kept_extra(policy))
     if w.kind == "h2o":
         sc = O.h2o_batch(ob, qw_bits, k_bits, units=units)
         pooled = sc
@@ -739,7 +746,7 @@ def main(argv=None):
     ap.add_argument("--score", choices=["snapkv", "quest"], default="snapkv",
                     help="score of the SnapKV workloads: windowed mass, or the Quest page bound")
     ap.add_argument("--page", type=int, default=16, help="tokens per page of the Quest bound")
-    ap.add_argument("--policy", choices=["quota", "global", "fair", "slack"], default="quota",
+    ap.add_argument("--policy", choices=["quota", "global", "fair", "slack", "ceil"], default="quota",
                     help="budget split: role quotas (the method), plain top-k, fair eviction, or "
                          "role quotas with the slack of saturated buckets filled by score")
     ap.add_argument("--keep-last", type=int, default=0,

@@ -37,11 +37,16 @@
  *   sequence s at columns cu[s] .. cu[s+1]-1.
  * Role arrays (uint8, one label per token, shared by all layers and heads).
  *   Dense: [b][n_max].  Varlen: [T].
- * Kept-index arrays (int32).  Sequence s keeps K_s = rolekv_kept_count(len_s,
- *   B) slots.  Dense: [L][b][Hkv][K], K = rolekv_kept_count(n_max, B).
- *   Varlen: [L][Hkv][Ktot], sequence s at offset cu_kept[s] = sum of K_s' for
- *   s' < s.  Kept positions are written in ascending order; when fewer than K_s
- *   tokens are eligible the tail of the row is -1.
+ * Kept-index arrays (int32).  Sequence s has a row of K_s =
+ *   rolekv_kept_rows(len_s, B, kept_extra) slots: its ceil(B*len_s) budget
+ *   plus the batch's kept_extra, at most len_s (kept_extra is 0 except for the
+ *   ceiling policy, whose total may exceed the budget).  Dense: [L][b][Hkv][K],
+ *   K = rolekv_kept_rows(n_max, B, kept_extra).  Varlen: [L][Hkv][Ktot],
+ *   sequence s at offset cu_kept[s] = sum of K_s' for s' < s.  Kept positions
+ *   are written in ascending order; the slots after the last kept position
+ *   (fewer eligible tokens than the budget, or the unused part of kept_extra)
+ *   hold -1.  kv_compact, decode_attention and rolekv_compress use the same
+ *   rows for the same batch and budget.
  * Batches without tokens.  When n_max is 0 or every sequence is empty, the
  *   buffers sized by tokens or kept slots are empty and may be NULL; the
  *   calls still write what is not empty: zero per-role kept counts and zero
@@ -80,6 +85,7 @@ extern "C" {
 #define ROLEKV_POLICY_GLOBAL 1      /* plain top-k, optional role ban (Sec. 4) */
 #define ROLEKV_POLICY_FAIR 2        /* equal retention rate per role (Sec. 5)  */
 #define ROLEKV_POLICY_SLACK 3       /* slack of saturated buckets by score     */
+#define ROLEKV_POLICY_CEIL 4        /* Algorithm 1's ceilings taken literally  */
 
 #define ROLEKV_MAX_ROLES 8
 #define ROLEKV_SELECT_MAX_N 40960   /* largest sequence role_alloc_select takes */
@@ -94,6 +100,9 @@ typedef struct rolekv_batch {
   int32_t n_max;
   const int32_t* seqlens_host;   /* [b] on the host, or NULL (dense)          */
   const int32_t* cu_seqlens_dev; /* [b+1] on the device, varlen only          */
+  int32_t kept_extra;            /* kept-row slots beyond ceil(B*n), >= 0;
+                                    ROLEKV_POLICY_CEIL needs at least the
+                                    number of weighted roles - 1; 0 otherwise */
 } rolekv_batch;
 
 /* Role-conditional allocation parameters (Section 4.1, Algorithm 1).
@@ -123,6 +132,14 @@ typedef struct rolekv_batch {
  *              buckets leave go to the highest-scoring tokens of the
  *              eligible buckets not kept yet (ties to the lower index); the
  *              total is the same min(ceil(B*n), eligible tokens).
+ *              ROLEKV_POLICY_CEIL: Algorithm 1's "top ceil(alpha_r B n_kv)
+ *              per bucket" taken literally: the ROLE_QUOTA water-filling of
+ *              saturated buckets, then each unsaturated bucket keeps the
+ *              ceiling of its share instead of floor plus largest remainder.
+ *              The total lies between min(ceil(B*n), eligible) and that plus
+ *              (unsaturated buckets - 1), so the batch's kept_extra must be at
+ *              least (roles with a positive weight, not banned) - 1, else the
+ *              call returns ROLEKV_ERR_INVALID_ARG.
  *   ban_mask   bit r set: role r keeps nothing.
  *   keep_last  recency floor (SnapKV's observation window, Section 7): the
  *              last R = min(keep_last, n, ceil(B*n)) tokens of each sequence
@@ -145,6 +162,11 @@ typedef struct rolekv_select_params {
 /* Number of kept slots of an n-token sequence at budget B: ceil(B*n) with B in
  * 1e-6 fixed point; -1 if B is outside (0, 1] or n < 0. */
 int64_t rolekv_kept_count(int64_t n, float budget);
+
+/* Width of an n-token sequence's kept-index row: min(n, rolekv_kept_count(n,
+ * budget) + kept_extra); -1 for a budget outside (0, 1], n < 0 or
+ * kept_extra < 0. */
+int64_t rolekv_kept_rows(int64_t n, float budget, int32_t kept_extra);
 
 /* Bytes of device workspace snapkv_score / h2o_score / rolekv_compress need for
  * this batch (op: 0 snapkv_score, 1 h2o_score, 2 rolekv_compress; W the SnapKV
@@ -221,8 +243,8 @@ int quest_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k,
  * compacted cache realises the 1-B memory and decode-time reduction).  For
  * every (layer, sequence, KV head) and each of its G query heads,
  *   out_g = sum_j softmax_j(scale * q_g . k_j) v_j
- * over the unit's rows j < ceil(budget * n) of k_cache / v_cache, skipping the
- * rows whose keep_idx entry is -1 (the padding of an infeasible budget).
+ * over the unit's rows j < rolekv_kept_rows(n, budget, kept_extra) of k_cache /
+ * v_cache, skipping the rows whose keep_idx entry is -1 (padding).
  *   q        bf16 decode queries, one token per sequence: [L][b][Hq][d]
  *            (s_tok is ignored).
  *   k_cache, v_cache  bf16 cache rows: kv_compact's output (dense

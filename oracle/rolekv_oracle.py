@@ -52,7 +52,8 @@ stride 1, same length, truncated at the sequence edges; "renormalized per
 bucket" = alpha_r / sum of alpha over the eligible buckets (alpha_r > 0 and
 n_r > 0) of the sequence; the total kept is exactly ceil(B n) (or all
 eligible tokens when fewer), apportioned by integer water-filling plus
-largest remainder; ties in score go to the lower token index; kept indices
+largest remainder (the CEIL split alone takes Algorithm 1's ceilings
+literally and may keep a few more); ties in score go to the lower token index; kept indices
 are returned in ascending position order.  Budgets and alphas are taken to
 fixed point with six decimals so that ceilings are exact.
 """

@@ -46,14 +46,14 @@ __global__ void __launch_bounds__(kThreads) compact_kernel(const CompactArgs a, 
     if (threadIdx.x < 32) {
       int64_t part = 0;
       for (int x = threadIdx.x; x < s; x += 32)
-        part += kept_slots(a.cu_seqlens[x + 1] - a.cu_seqlens[x], a.budget_fx);
+        part += kept_rows(a.cu_seqlens[x + 1] - a.cu_seqlens[x], a.budget_fx, a.kept_extra);
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
       if (threadIdx.x == 0) cu_kept = part;
     }
     __syncthreads();
     kbase = (static_cast<int64_t>(l) * a.Hkv + h) * a.Ktot + cu_kept;
-    K_s = kept_slots(n, a.budget_fx);
+    K_s = kept_rows(n, a.budget_fx, a.kept_extra);
   } else {
     tok0 = 0;
     n = a.n_max;

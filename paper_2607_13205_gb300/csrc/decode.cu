@@ -47,7 +47,7 @@ __device__ __forceinline__ int64_t kept_prefix(const DecodeArgs& a, int s) {
   // kept rows of the sequences before s (varlen), by one warp
   int64_t part = 0;
   for (int x = threadIdx.x & 31; x < s; x += 32)
-    part += kept_slots(a.cu_seqlens[x + 1] - a.cu_seqlens[x], a.budget_fx);
+    part += kept_rows(a.cu_seqlens[x + 1] - a.cu_seqlens[x], a.budget_fx, a.kept_extra);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
   return part;
@@ -113,7 +113,7 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const Decod
     n = a.n_max;
     row0 = 0;
   }
-  const int m = static_cast<int>(kept_slots(n, a.budget_fx));
+  const int m = static_cast<int>(kept_rows(n, a.budget_fx, a.kept_extra));
   const int r0 = split * a.rows_per_split;
   if (r0 >= m) return;                              // (uniform: no partial is read)
   const int r1 = (m - r0 < a.rows_per_split) ? m : r0 + a.rows_per_split;
@@ -352,7 +352,7 @@ __global__ void __launch_bounds__(256) decode_combine_kernel(const DecodeArgs a)
   const int s = (u / a.Hkv) % a.b;
   const int l = u / (a.Hkv * a.b);
   const int n = a.varlen ? a.cu_seqlens[s + 1] - a.cu_seqlens[s] : a.n_max;
-  const int m = static_cast<int>(kept_slots(n, a.budget_fx));
+  const int m = static_cast<int>(kept_rows(n, a.budget_fx, a.kept_extra));
   const int ns = (m + a.rows_per_split - 1) / a.rows_per_split;
   const float* base = a.part + (static_cast<int64_t>(u) * a.n_splits * a.G + g) * (a.d + 2);
   const int64_t stride = static_cast<int64_t>(a.G) * (a.d + 2);

@@ -73,6 +73,7 @@ struct SelectArgs {
   int32_t n_roles;
   int64_t alpha_fx[ROLEKV_MAX_ROLES];   // fixed-point weights, 0 for banned roles
   int64_t budget_fx;
+  int32_t kept_extra;                   // kept-row width beyond ceil(B n)
   int32_t policy;
   uint32_t ban_mask;
   int32_t keep_last;                    // recency floor (tokens), 0 = none
@@ -110,7 +111,8 @@ struct DecodeArgs {
   int32_t varlen;
   const int32_t* cu_seqlens;
   int32_t n_units;
-  int64_t budget_fx;                // rows of a sequence: kept_slots(n, budget_fx)
+  int64_t budget_fx;                // rows of a sequence: kept_rows(n, budget_fx, kept_extra)
+  int32_t kept_extra;
   int64_t Ktot;                     // packed rows per (layer, head), varlen
   int32_t K_dense;                  // rows per unit, dense
   const uint16_t* q;                // decode queries [L][b][Hq][d] (strides below)
@@ -141,6 +143,7 @@ struct CompactArgs {
   int32_t K_dense;
   int32_t K_max;                    // widest kept row (grid sizing)
   int64_t budget_fx;
+  int32_t kept_extra;
   const int32_t* cu_seqlens;
   int32_t n_units;
   const uint16_t* k;
@@ -161,6 +164,13 @@ constexpr int64_t kFixedOne = 1000000;
 
 __host__ __device__ inline int64_t kept_slots(int64_t n, int64_t budget_fx) {
   return (budget_fx * n + kFixedOne - 1) / kFixedOne;
+}
+
+// Width of an n-token sequence's kept row: ceil(B n) slots plus `extra` (room
+// for the ceiling split's overshoot), at most n.
+__host__ __device__ inline int64_t kept_rows(int64_t n, int64_t budget_fx, int32_t extra) {
+  const int64_t k = kept_slots(n, budget_fx) + extra;
+  return k < n ? k : n;
 }
 
 }  // namespace rolekv

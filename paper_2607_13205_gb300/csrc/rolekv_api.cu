@@ -60,6 +60,7 @@ size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
 struct BatchInfo {
   int L, b, Hq, Hkv, G, d, n_max;
+  int kept_extra;
   bool varlen;
   int64_t T;
   int64_t n_units;
@@ -72,6 +73,8 @@ int check_batch(const rolekv_batch* bt, BatchInfo* bi) {
                 bt->L, bt->b, bt->Hq, bt->Hkv, bt->d, bt->n_max);
   if (bt->Hq % bt->Hkv != 0)
     return fail(ROLEKV_ERR_INVALID_ARG, "Hq=%d is not a multiple of Hkv=%d", bt->Hq, bt->Hkv);
+  if (bt->kept_extra < 0) return fail(ROLEKV_ERR_INVALID_ARG, "kept_extra=%d must be >= 0", bt->kept_extra);
+  bi->kept_extra = bt->kept_extra;
   bi->L = bt->L;
   bi->b = bt->b;
   bi->Hq = bt->Hq;
@@ -345,11 +348,12 @@ void fill_compact(const BatchInfo& bi, const int32_t* cu_seqlens, int64_t budget
   a->n_max = bi.n_max;
   a->varlen = bi.varlen;
   a->budget_fx = budget_fx;
-  a->K_dense = static_cast<int32_t>(kept_slots(bi.n_max, budget_fx));
+  a->kept_extra = bi.kept_extra;
+  a->K_dense = static_cast<int32_t>(kept_rows(bi.n_max, budget_fx, bi.kept_extra));
   a->K_max = a->K_dense;
   a->Ktot = 0;
   if (bi.varlen)
-    for (int s = 0; s < bi.b; ++s) a->Ktot += kept_slots(seqlens_host[s], budget_fx);
+    for (int s = 0; s < bi.b; ++s) a->Ktot += kept_rows(seqlens_host[s], budget_fx, bi.kept_extra);
   a->cu_seqlens = cu_seqlens;
   a->n_units = static_cast<int32_t>(bi.n_units);
   a->k = static_cast<const uint16_t*>(k.ptr);
@@ -393,7 +397,8 @@ int fill_select(const BatchInfo& bi, const rolekv_batch* bt, const rolekv_select
   if (!(sp->budget > 0.f) || sp->budget > 1.f)
     return fail(ROLEKV_ERR_INVALID_ARG, "budget %g outside (0, 1]", static_cast<double>(sp->budget));
   if (sp->policy != ROLEKV_POLICY_ROLE_QUOTA && sp->policy != ROLEKV_POLICY_GLOBAL &&
-      sp->policy != ROLEKV_POLICY_FAIR && sp->policy != ROLEKV_POLICY_SLACK)
+      sp->policy != ROLEKV_POLICY_FAIR && sp->policy != ROLEKV_POLICY_SLACK &&
+      sp->policy != ROLEKV_POLICY_CEIL)
     return fail(ROLEKV_ERR_INVALID_ARG, "unknown policy %d", sp->policy);
   if (sp->keep_last < 0) return fail(ROLEKV_ERR_INVALID_ARG, "keep_last=%d must be >= 0", sp->keep_last);
   if (sp->key_role >= sp->n_roles) return fail(ROLEKV_ERR_INVALID_ARG, "key_role %d >= n_roles", sp->key_role);
@@ -420,10 +425,21 @@ int fill_select(const BatchInfo& bi, const rolekv_batch* bt, const rolekv_select
       return fail(ROLEKV_ERR_INVALID_ARG, "alpha[%d]=%g must be finite and >= 0", r, static_cast<double>(al));
     a->alpha_fx[r] = ((sp->ban_mask >> r) & 1u) ? 0 : to_fixed(al);
   }
-  a->K_dense = static_cast<int32_t>(kept_slots(bi.n_max, a->budget_fx));
+  if (sp->policy == ROLEKV_POLICY_CEIL) {
+    // the ceilings of the unsaturated buckets' shares overshoot the budget by
+    // less than one slot each, and at least one bucket takes a whole share
+    int weighted = 0;
+    for (int r = 0; r < sp->n_roles; ++r) weighted += a->alpha_fx[r] > 0;
+    if (bi.kept_extra < weighted - 1)
+      return fail(ROLEKV_ERR_INVALID_ARG,
+                  "the ceiling policy over %d weighted roles needs batch kept_extra >= %d (got %d)",
+                  weighted, weighted - 1, bi.kept_extra);
+  }
+  a->kept_extra = bi.kept_extra;
+  a->K_dense = static_cast<int32_t>(kept_rows(bi.n_max, a->budget_fx, bi.kept_extra));
   a->Ktot = 0;
   if (bi.varlen)
-    for (int s = 0; s < bi.b; ++s) a->Ktot += kept_slots(bt->seqlens_host[s], a->budget_fx);
+    for (int s = 0; s < bi.b; ++s) a->Ktot += kept_rows(bt->seqlens_host[s], a->budget_fx, bi.kept_extra);
   return ROLEKV_OK;
 }
 
@@ -477,9 +493,14 @@ int64_t rolekv_kept_count(int64_t n, float budget) {
   return kept_slots(n, to_fixed(budget));
 }
 
+int64_t rolekv_kept_rows(int64_t n, float budget, int32_t kept_extra) {
+  if (n < 0 || kept_extra < 0 || !(budget > 0.f) || budget > 1.f) return -1;
+  return kept_rows(n, to_fixed(budget), kept_extra);
+}
+
 const char* rolekv_last_error(void) { return g_err; }
 
-const char* rolekv_version(void) { return "rolekv 0.1 (sm_103a)"; }
+const char* rolekv_version(void) { return "rolekv 0.2 (sm_103a)"; }
 
 int rolekv_selftest_wait(int64_t limit_ns, int32_t* status_dev, void* stream) {
   if (status_dev == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "status_dev is NULL");
@@ -685,12 +706,12 @@ void decode_rows(const BatchInfo& bi, const rolekv_batch* bt, int64_t bfx, int64
   *total = 0;
   if (bi.varlen) {
     for (int s = 0; s < bi.b; ++s) {
-      const int64_t m = kept_slots(bt->seqlens_host[s], bfx);
+      const int64_t m = kept_rows(bt->seqlens_host[s], bfx, bi.kept_extra);
       *m_max = m > *m_max ? m : *m_max;
       *total += m;
     }
   } else {
-    *m_max = kept_slots(bi.n_max, bfx);
+    *m_max = kept_rows(bi.n_max, bfx, bi.kept_extra);
     *total = *m_max * bi.b;
   }
 }
@@ -757,6 +778,7 @@ int decode_attention(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k
   a.cu_seqlens = batch->cu_seqlens_dev;
   a.n_units = static_cast<int32_t>(bi.n_units);
   a.budget_fx = bfx;
+  a.kept_extra = bi.kept_extra;
   a.Ktot = bi.varlen ? total : 0;
   a.K_dense = bi.varlen ? 0 : static_cast<int32_t>(m_max);
   a.q = static_cast<const uint16_t*>(q.ptr);

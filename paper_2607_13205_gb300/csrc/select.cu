@@ -216,7 +216,8 @@ __device__ __forceinline__ void pass1(const UnitView& v, int n_roles, uint32_t b
 
 // Quotas of one sequence by warp 0, lane r for role r: water-filling of the
 // weights over the role counts, then the integer remainders to the largest
-// fractional parts (ties to the lower role), the arithmetic stated in rolekv.h.
+// fractional parts (ties to the lower role), or under CEIL the ceiling of each
+// share; the arithmetic stated in rolekv.h.
 __device__ __forceinline__ int64_t sum8(int64_t v) {
   v += __shfl_xor_sync(0xffffffffu, v, 1);
   v += __shfl_xor_sync(0xffffffffu, v, 2);
@@ -261,20 +262,26 @@ __device__ void quotas_warp(const SelectArgs& a, int lane, int64_t K_full, SelSh
       left -= sum8(sat ? cnt : 0);
     }
     const int64_t A = sum8(live ? alpha : 0);
-    int64_t rem = -1;
-    if (live && A != 0) {
-      q = alpha * left / A;
-      rem = alpha * left % A;
-    }
-    const int64_t extra = left - sum8(live ? q : 0);
-    int rank = 0;
+    if (a.policy == ROLEKV_POLICY_CEIL) {
+      // Algorithm 1 read literally: each unsaturated bucket takes the ceiling
+      // of its share (the total may exceed the budget; the rows are wider)
+      if (live && A != 0) q = (alpha * left + A - 1) / A;
+    } else {
+      int64_t rem = -1;
+      if (live && A != 0) {
+        q = alpha * left / A;
+        rem = alpha * left % A;
+      }
+      const int64_t extra = left - sum8(live ? q : 0);
+      int rank = 0;
 #pragma unroll
-    for (int x = 0; x < kR; ++x) {
-      const int64_t rx = __shfl_sync(0xffffffffu, rem, x);
-      const int lx = __shfl_sync(0xffffffffu, static_cast<int>(live), x);
-      if (lx && (rx > rem || (rx == rem && x < r))) ++rank;
+      for (int x = 0; x < kR; ++x) {
+        const int64_t rx = __shfl_sync(0xffffffffu, rem, x);
+        const int lx = __shfl_sync(0xffffffffu, static_cast<int>(live), x);
+        if (lx && (rx > rem || (rx == rem && x < r))) ++rank;
+      }
+      if (live && A != 0 && rank < extra) q += 1;
     }
-    if (live && A != 0 && rank < extra) q += 1;
     if (a.policy == ROLEKV_POLICY_SLACK) {
       q = q < cnt ? q : cnt;
       const int64_t slack = k_all - sum8(q);
@@ -500,7 +507,8 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
   const int64_t sbase =
       a.varlen ? (static_cast<int64_t>(l) * a.Hkv + h) * a.T + tok0 : static_cast<int64_t>(u) * a.n_max;
   const int64_t rbase = a.varlen ? tok0 : static_cast<int64_t>(s) * a.n_max;
-  const int64_t K_s = kept_slots(n, a.budget_fx);
+  const int64_t K_s = kept_slots(n, a.budget_fx);              // the budget
+  const int64_t width = kept_rows(n, a.budget_fx, a.kept_extra); // the kept row
 
   UnitView v;
   v.sp = a.scores + sbase;
@@ -553,7 +561,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
     int64_t part = 0;
     if (a.varlen) {
       for (int x = tid; x < s; x += NT)
-        part += kept_slots(a.cu_seqlens[x + 1] - a.cu_seqlens[x], a.budget_fx);
+        part += kept_rows(a.cu_seqlens[x + 1] - a.cu_seqlens[x], a.budget_fx, a.kept_extra);
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
@@ -1001,7 +1009,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
       if (count_roles) kr += shl64(1ull, 8u * __ldg(v.rp + t));
     }
   }, S.warp_tot);
-  for (int64_t j = total + tid; j < K_s; j += NT) dst[j] = -1;
+  for (int64_t j = total + tid; j < width; j += NT) dst[j] = -1;
 
   if (a.keep_mask != nullptr) {
     uint8_t* mp = a.keep_mask + sbase;

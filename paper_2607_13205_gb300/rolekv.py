@@ -18,7 +18,7 @@ _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "librolekv.
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA = 0, 1, 2, 3, 4
 STATUS_NONFINITE, STATUS_BAD_INDEX, STATUS_TIMEOUT = 1, 2, 4
-POLICY_ROLE_QUOTA, POLICY_GLOBAL, POLICY_FAIR, POLICY_SLACK = 0, 1, 2, 3
+POLICY_ROLE_QUOTA, POLICY_GLOBAL, POLICY_FAIR, POLICY_SLACK, POLICY_CEIL = 0, 1, 2, 3, 4
 MAX_ROLES = 8
 SELECT_MAX_N = 40960
 OP_SNAPKV, OP_H2O, OP_COMPRESS = 0, 1, 2
@@ -39,7 +39,7 @@ class BatchDesc(ctypes.Structure):
     _fields_ = [("L", ctypes.c_int32), ("b", ctypes.c_int32), ("Hq", ctypes.c_int32),
                 ("Hkv", ctypes.c_int32), ("d", ctypes.c_int32), ("n_max", ctypes.c_int32),
                 ("seqlens_host", ctypes.POINTER(ctypes.c_int32)),
-                ("cu_seqlens_dev", ctypes.c_void_p)]
+                ("cu_seqlens_dev", ctypes.c_void_p), ("kept_extra", ctypes.c_int32)]
 
 
 class SelectParams(ctypes.Structure):
@@ -54,6 +54,7 @@ _lib = None
 # (name, restype, argtypes) of every exported function
 _SIGNATURES = [
     ("rolekv_kept_count", ctypes.c_int64, [ctypes.c_int64, ctypes.c_float]),
+    ("rolekv_kept_rows", ctypes.c_int64, [ctypes.c_int64, ctypes.c_float, ctypes.c_int32]),
     ("rolekv_workspace_size", ctypes.c_int,
      [ctypes.c_int, ctypes.POINTER(BatchDesc), ctypes.c_int32, ctypes.POINTER(ctypes.c_size_t)]),
     ("snapkv_score", ctypes.c_int,
@@ -132,11 +133,13 @@ def _stream(stream=None):
 
 class Batch:
     """Shapes of one call.  seqlens (list of ints) makes it a varlen batch; the
-    device copy of the prefix sums is created here, once."""
+    device copy of the prefix sums is created here, once.  kept_extra widens
+    every kept row beyond ceil(B n) (the ceiling policy needs it)."""
 
     def __init__(self, L, b, Hq, Hkv, d, n_max, seqlens: Optional[Sequence[int]] = None,
-                 device="cuda"):
+                 device="cuda", kept_extra: int = 0):
         self.L, self.b, self.Hq, self.Hkv, self.d, self.n_max = L, b, Hq, Hkv, d, n_max
+        self.kept_extra = int(kept_extra)
         self.seqlens = list(seqlens) if seqlens is not None else None
         self._host = None
         self.cu_seqlens = None
@@ -148,7 +151,8 @@ class Batch:
             self.cu_seqlens = torch.tensor(cu, dtype=torch.int32, device=device)
         self.desc = BatchDesc(L, b, Hq, Hkv, d, n_max,
                               self._host if self._host is not None else None,
-                              ctypes.c_void_p(self.cu_seqlens.data_ptr()) if self.cu_seqlens is not None else None)
+                              ctypes.c_void_p(self.cu_seqlens.data_ptr()) if self.cu_seqlens is not None else None,
+                              self.kept_extra)
 
     @property
     def varlen(self) -> bool:
@@ -170,8 +174,8 @@ class Batch:
 
     def kept_shape(self, budget: float):
         if self.varlen:
-            return (self.L, self.Hkv, sum(kept_count(n, budget) for n in self.seqlens))
-        return (self.L, self.b, self.Hkv, kept_count(self.n_max, budget))
+            return (self.L, self.Hkv, sum(kept_rows(n, budget, self.kept_extra) for n in self.seqlens))
+        return (self.L, self.b, self.Hkv, kept_rows(self.n_max, budget, self.kept_extra))
 
 
 def tensor_desc(t: torch.Tensor, packed: bool = False) -> Tensor:
@@ -203,6 +207,10 @@ def select_params(budget: float, alpha: Sequence[float], alpha_key: float = 0.0,
 
 def kept_count(n: int, budget: float) -> int:
     return int(lib().rolekv_kept_count(int(n), float(budget)))
+
+
+def kept_rows(n: int, budget: float, kept_extra: int = 0) -> int:
+    return int(lib().rolekv_kept_rows(int(n), float(budget), int(kept_extra)))
 
 
 def workspace_size(op: int, batch: Batch, W: int = 0) -> int:

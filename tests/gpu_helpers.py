@@ -26,13 +26,14 @@ def assert_scores_close(got: np.ndarray, ref: np.ndarray, what: str = ""):
                            f"ref={ref[bad[0]]!r} rel={err[bad[0]] / max(abs(ref[bad[0]]), 1e-300):.3g}")
 
 
-def oracle_batch(w: I.Workload) -> O.Batch:
-    return O.Batch(w.L, w.b, w.Hq, w.Hkv, w.d, w.n, seqlens=list(w.seqlens) if w.varlen else None)
+def oracle_batch(w: I.Workload, kept_extra: int = 0) -> O.Batch:
+    return O.Batch(w.L, w.b, w.Hq, w.Hkv, w.d, w.n, seqlens=list(w.seqlens) if w.varlen else None,
+                   kept_extra=kept_extra)
 
 
-def lib_batch(w: I.Workload, device) -> R.Batch:
+def lib_batch(w: I.Workload, device, kept_extra: int = 0) -> R.Batch:
     return R.Batch(w.L, w.b, w.Hq, w.Hkv, w.d, w.n, seqlens=list(w.seqlens) if w.varlen else None,
-                   device=device)
+                   device=device, kept_extra=kept_extra)
 
 
 def check_index_sets(ob: O.Batch, u: int, got_idx: np.ndarray, ref_scores: np.ndarray, roles_np,

@@ -53,6 +53,16 @@ def test_kept_count_matches_oracle(lib):
     assert R.kept_count(-1, 0.5) == -1
 
 
+def test_kept_rows_matches_oracle(lib):
+    for extra in (0, 1, 3, 7, 100000):
+        ob = O.Batch(1, 1, 1, 1, 8, 1, kept_extra=extra)
+        for n in (0, 1, 7, 100, 2048, 32768, 123457):
+            for b in (0.05, 0.1, 0.333, 1.0):
+                assert R.kept_rows(n, b, extra) == ob.kept_rows(n, b), (n, b, extra)
+    assert R.kept_rows(10, 0.5, -1) == -1
+    assert R.kept_rows(10, 0.0, 2) == -1
+
+
 def _batch(**kw):
     d = dict(L=2, b=3, Hq=8, Hkv=2, d=128, n_max=1000)
     d.update(kw)
@@ -99,9 +109,19 @@ def test_host_rejects_bad_arguments(lib):
     p_neg = R.select_params(0.1, [0.25, 0.0, -0.7, 0.05])
     rc = lib.role_alloc_select(ctypes.byref(b), f, f, ctypes.byref(p_neg), 1, f, None, None, None, None)
     assert rc == R.ERR_INVALID_ARG
-    p_pol = R.select_params(0.1, [0.25, 0.0, 0.7, 0.05], policy=4)
+    p_pol = R.select_params(0.1, [0.25, 0.0, 0.7, 0.05], policy=5)
     rc = lib.role_alloc_select(ctypes.byref(b), f, f, ctypes.byref(p_pol), 1, f, None, None, None, None)
     assert rc == R.ERR_INVALID_ARG                                      # unknown policy
+    # the ceiling policy over 3 weighted roles needs rows 2 slots wider
+    p_ceil = R.select_params(0.1, [0.25, 0.0, 0.7, 0.05], policy=R.POLICY_CEIL)
+    narrow = _batch()
+    narrow.kept_extra = 1
+    rc = lib.role_alloc_select(ctypes.byref(narrow), f, f, ctypes.byref(p_ceil), 1, f, None, None, None, None)
+    assert rc == R.ERR_INVALID_ARG and b"kept_extra >= 2" in lib.rolekv_last_error()
+    neg = _batch()
+    neg.kept_extra = -1
+    rc = lib.kv_compact(ctypes.byref(neg), t, t, f, 0.1, f, f, None, None)
+    assert rc == R.ERR_INVALID_ARG and b"kept_extra" in lib.rolekv_last_error()
     p_floor = R.select_params(0.1, [0.25, 0.0, 0.7, 0.05], keep_last=-1)
     rc = lib.role_alloc_select(ctypes.byref(b), f, f, ctypes.byref(p_floor), 1, f, None, None, None, None)
     assert rc == R.ERR_INVALID_ARG                                      # negative floor

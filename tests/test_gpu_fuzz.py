@@ -1,6 +1,6 @@
 """Seeded sweep over shapes: random small configurations (head dim, GQA group,
 window, pool width, length mix with empty and very short sequences, budget,
-policy, recency floor), each taken through score -> select -> compact ->
+policy, recency floor, kept-row widening), each taken through score -> select -> compact ->
 decode on the GPU and compared with the fp64 oracle: scores within 1e-3
 relative, selection and compaction bit-exact on the kernel's own scores,
 decode within the decode tolerance; half of them also through the H2O score
@@ -38,21 +38,24 @@ def _config(seed):
     w = I.WORKLOADS["tiny"].scaled(L=1, b=b, Hq=G * Hkv, Hkv=Hkv, d=d, n=n, W=W,
                                    pool_k=int(g.choice([1, 3, 5, 7, 15])), seqlens=seqlens)
     B = float(g.choice([0.01, 0.05, 0.1, 0.3, 0.5, 1.0]))
-    policy = int(g.integers(0, 4))
+    policy = int(g.integers(0, 5))
     keep_last = int(g.choice([0, 0, 4, 40]))
     akey = float(g.choice([0.0, 0.02]))
     ban = int(1 << I.ROLE_KEY) if g.random() < 0.2 else 0
-    return w, B, policy, keep_last, akey, ban
+    extra = int(g.choice([0, 0, 0, 2]))
+    if policy == R.POLICY_CEIL:
+        extra = I.N_ROLES - 1 + extra
+    return w, B, policy, keep_last, akey, ban, extra
 
 
 @pytest.mark.parametrize("seed", list(range(N_CASES)))
 def test_random_configuration_end_to_end(seed):
-    w, B, policy, keep_last, akey, ban = _config(seed)
+    w, B, policy, keep_last, akey, ban, extra = _config(seed)
     roles_np = I.workload_roles(w, seed)
     K, V = I.make_kv(w, roles_np, seed, device=DEV)
     qw = I.make_q_window(w, seed, device=DEV)
-    batch = lib_batch(w, DEV)
-    ob = oracle_batch(w)
+    batch = lib_batch(w, DEV, kept_extra=extra)
+    ob = oracle_batch(w, kept_extra=extra)
     status = torch.zeros(1, dtype=torch.int32, device=DEV)
 
     scores = torch.full(batch.score_shape(), -1.0, dtype=torch.float32, device=DEV)
@@ -117,7 +120,7 @@ def test_random_configuration_end_to_end(seed):
 def test_random_configuration_h2o_and_quest(seed):
     """The same seeded configurations through the H2O score (every causal
     query, n kept at most 1500 for the oracle) and the Quest page bound."""
-    w, B, policy, keep_last, akey, ban = _config(seed)
+    w, B, policy, keep_last, akey, ban, _ = _config(seed)
     if w.n > 1500:
         w = w.scaled(n=1500, seqlens=None if w.seqlens is None else tuple(min(x, 1500) for x in w.seqlens))
     roles_np = I.workload_roles(w, seed)

@@ -323,6 +323,15 @@ SELECT_CASES = [
     ("slack_floor_mid_n", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=12001), 0.20, 0.02, R.POLICY_SLACK, 0, 7, 64),
     ("slack_ban_max_n", _w("long", L=1, b=1, Hq=4, Hkv=1, n=R.SELECT_MAX_N), 0.30, 0.02, R.POLICY_SLACK,
      1 << I.ROLE_KEY, 1),
+    # Algorithm 1's per-bucket ceilings taken literally (rows widened by
+    # kept_extra = N_ROLES - 1 unless given), and widened rows under the exact split
+    ("ceil_b10_pool7", _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=5000), 0.10, 0.02, R.POLICY_CEIL, 0, 7),
+    ("ceil_varlen_floor32", VARLEN4, 0.05, 0.0, R.POLICY_CEIL, 0, 7, 32),
+    ("ceil_ban_max_n", _w("long", L=1, b=1, Hq=4, Hkv=1, n=R.SELECT_MAX_N), 0.30, 0.02, R.POLICY_CEIL,
+     1 << I.ROLE_KEY, 1),
+    ("ceil_full_budget", _w("llama8b", L=1, b=1, Hq=4, Hkv=1, n=777), 1.0, 0.02, R.POLICY_CEIL, 0, 3),
+    ("ceil_mid_n_extra9", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=12001), 0.20, 0.02, R.POLICY_CEIL, 0, 7, 0, 9),
+    ("quota_varlen_extra5", VARLEN4, 0.10, 0.02, 0, 0, 7, 0, 5),
 ]
 
 
@@ -330,8 +339,9 @@ SELECT_CASES = [
 def test_role_alloc_select_bit_exact(case):
     name, w, B, akey, policy, ban, pool_k = case[:7]
     keep_last = case[7] if len(case) > 7 else 0
+    extra = case[8] if len(case) > 8 else (I.N_ROLES - 1 if policy == R.POLICY_CEIL else 0)
     roles_np = I.workload_roles(w, 2)
-    batch = lib_batch(w, DEV)
+    batch = lib_batch(w, DEV, kept_extra=extra)
     scores = _tied_scores(batch.score_shape(), 5)
     roles = torch.as_tensor(roles_np, device=DEV)
     params = R.select_params(B, I.PAPER_ALPHA, alpha_key=akey, key_role=I.ROLE_KEY, policy=policy,
@@ -344,7 +354,7 @@ def test_role_alloc_select_bit_exact(case):
                         kept_per_role=per_role, status=status)
     torch.cuda.synchronize()
     assert int(status.item()) == 0
-    ob = oracle_batch(w)
+    ob = oracle_batch(w, kept_extra=extra)
     sc = scores.cpu().numpy()
     unit_scores = {}
     for u in range(ob.n_units):
@@ -551,16 +561,18 @@ def test_kv_compact_bit_exact(varlen):
 
 # ------------------------------------------------------------- whole pipeline
 
-@pytest.mark.parametrize("name", ["tiny", "ragged_small"])
+@pytest.mark.parametrize("name", ["tiny", "ragged_small", "ragged_small_ceil"])
 def test_rolekv_compress_pipeline(name):
     if name == "tiny":
         w = I.WORKLOADS["tiny"]
     else:
         w = _w("ragged", L=2, b=4, Hq=14, Hkv=2, n=3000, seqlens=(3000, 1024, 77, 2222))
     B = w.budgets[0]
+    policy = R.POLICY_CEIL if name.endswith("ceil") else R.POLICY_ROLE_QUOTA
+    extra = I.N_ROLES - 1 if policy == R.POLICY_CEIL else 0
     roles_np, K, V, qw = _snapkv_inputs(w, seed=6)
-    batch = lib_batch(w, DEV)
-    params = R.select_params(B, I.PAPER_ALPHA, 0.0, I.ROLE_KEY)
+    batch = lib_batch(w, DEV, kept_extra=extra)
+    params = R.select_params(B, I.PAPER_ALPHA, 0.0, I.ROLE_KEY, policy=policy)
     keep = torch.empty(batch.kept_shape(B), dtype=torch.int32, device=DEV)
     k_out = torch.empty(R.compact_shape(batch, B), dtype=torch.bfloat16, device=DEV)
     v_out = torch.empty_like(k_out)
@@ -574,7 +586,7 @@ def test_rolekv_compress_pipeline(name):
     R.role_alloc_select(batch, scores, roles, params, keep2)
     torch.cuda.synchronize()
     assert torch.equal(keep, keep2)
-    ob = oracle_batch(w)
+    ob = oracle_batch(w, kept_extra=extra)
     ref = O.snapkv_batch(ob, I.bf16_bits(qw), I.bf16_bits(K), w.W, w.pool_k)
     cu_kept = ob.kept_offsets(B)
     keep_np = keep.cpu().numpy()
@@ -588,7 +600,8 @@ def test_rolekv_compress_pipeline(name):
         else:
             row = keep_np.reshape(ob.n_units, -1)[u]
             kr = ko.reshape(ob.n_units, -1, w.d)[u]
-        check_index_sets(ob, u, row, pooled, roles_np, I.N_ROLES, I.PAPER_ALPHA, I.ROLE_KEY, 0.0, B)
+        check_index_sets(ob, u, row, pooled, roles_np, I.N_ROLES, I.PAPER_ALPHA, I.ROLE_KEY, 0.0, B,
+                         policy)
         assert np.array_equal(kr, O.compact_unit(ob.kv_rows(kb, u), row))
 
 

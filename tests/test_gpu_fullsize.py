@@ -120,6 +120,41 @@ def _check_sampled_snapkv(w, B, ob, units, r, alpha_key):
         assert np.array_equal(_unit_rows(ob, vo_all, u, kept_off), O.compact_unit(v.v[0, 0, 0], row))
 
 
+def _check_ceil_select(w, B, r, units):
+    """The literal ceiling split (rows N_ROLES - 1 slots wider) on the
+    kernel's own scores: bit-exact against the oracle on the sampled units;
+    on every unit the row is ascending, -1 padded, and keeps between
+    ceil(B n) and ceil(B n) + 3 tokens, counted per role."""
+    extra = I.N_ROLES - 1
+    batch = lib_batch(w, DEV, kept_extra=extra)
+    ob = oracle_batch(w, kept_extra=extra)
+    pre = torch.as_tensor(r["scores"], device=DEV)
+    params = R.select_params(B, I.PAPER_ALPHA, 0.0, I.ROLE_KEY, policy=R.POLICY_CEIL)
+    keep = torch.full(batch.kept_shape(B), -7, dtype=torch.int32, device=DEV)
+    per_role = torch.empty((batch.n_units, I.N_ROLES), dtype=torch.int32, device=DEV)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    R.role_alloc_select(batch, pre, torch.as_tensor(r["roles"], device=DEV), params, keep,
+                        pool_k=w.pool_k, kept_per_role=per_role, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    keep_np, pr = keep.cpu().numpy(), per_role.cpu().numpy()
+    kept_off = ob.kept_offsets(B)
+    for u in range(ob.n_units):
+        n = ob.seqlens[ob.unit(u)[1]]
+        row = _unit_rows(ob, keep_np, u, kept_off)
+        assert row.size == ob.kept_rows(n, B)
+        kept = row[row >= 0]
+        assert np.all(row[kept.size:] == -1) and np.all(np.diff(kept) > 0)
+        K = O.kept_count(n, B)
+        assert K <= kept.size <= K + extra and int(pr[u].sum()) == kept.size, (u, kept.size, K)
+    for u in units:
+        sc = O.maxpool1d(ob.score_view(r["scores"], u).astype(np.float64), w.pool_k)
+        idx, per = O.select_batch(ob, {u: sc}, r["roles"], I.N_ROLES, I.PAPER_ALPHA, I.ROLE_KEY, 0.0,
+                                  B, O.POLICY_CEIL)[u]
+        assert np.array_equal(_unit_rows(ob, keep_np, u, kept_off), idx), f"ceil unit {u}"
+        assert list(pr[u]) == per
+
+
 def test_long_context_full_size():
     """L=32, b=4, N=32768, 32/8 heads, d=128, W=64, pool 7, B=0.10 (~17 GB K/V)."""
     w = I.WORKLOADS["long"]
@@ -128,6 +163,7 @@ def test_long_context_full_size():
     ob = oracle_batch(w)
     _check_all_units(w, B, ob, r, 0.0, lambda n: min(w.W, n) * w.G)
     _check_sampled_snapkv(w, B, ob, [0, 517, ob.n_units - 1], r, 0.0)
+    _check_ceil_select(w, B, r, [0, 517, ob.n_units - 1])
 
 
 @pytest.mark.parametrize("B", I.WORKLOADS["llama8b"].budgets)

@@ -25,6 +25,7 @@
 // query blocks; a block's normalisers are its own, so they stay on chip).
 // attn_pass_kernel runs one pass per launch (the no-workspace SnapKV call).
 #include <cuda.h>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 #include <cmath>
@@ -736,7 +737,11 @@ struct FCfg {
   static constexpr int kPosOff = kLseOff + kRowsMax * 4;
   static constexpr int kRedOff = kPosOff + kRowsMax * 4;
   static constexpr int kMergeOff = kRedOff + (kParts - 1) * kTileKeys * 4;
-  static constexpr int kBarOff = kMergeOff + kParts * kRowsMax * 8;
+  // the extra pass-2 k-step: row normalisers (256 rows) against ones (128
+  // keys), 16 bf16 columns each, K-major without swizzle
+  static constexpr int kNlOff = kMergeOff + kParts * kRowsMax * 8;
+  static constexpr int kOnesOff = kNlOff + kRowsMax * 32;
+  static constexpr int kBarOff = kOnesOff + kTileKeys * 32;
   // k_full/k_empty[SK], q_full, q_empty, acc_full[2], acc_empty[2], merge_full,
   // red_full[2], red_empty[2], drain, pub, lse_go, lse_ready
   static constexpr int kNumBars = 2 * SK + 15;
@@ -748,6 +753,8 @@ struct FCfg {
 struct FShared {
   uint8_t* q;
   uint8_t* k;
+  uint8_t* nlb;      // [256 rows][16] bf16: -lse2_j / c1 in three parts, then zeros
+  uint8_t* ones;     // [128 keys][16] bf16: 1, 1, 1, then zeros
   float* lse;        // negated log2 normalisers of the current item's rows
   int32_t* pos;
   float* red;
@@ -771,6 +778,8 @@ __device__ __forceinline__ FShared fcarve(uint8_t* raw) {
   s.pos = reinterpret_cast<int32_t*>(base + C::kPosOff);
   s.red = reinterpret_cast<float*>(base + C::kRedOff);
   s.merge = reinterpret_cast<float2*>(base + C::kMergeOff);
+  s.nlb = base + C::kNlOff;
+  s.ones = base + C::kOnesOff;
   uint64_t* b = reinterpret_cast<uint64_t*>(base + C::kBarOff);
   s.k_full = b;
   s.k_empty = b + C::SK;
@@ -793,6 +802,21 @@ __device__ __forceinline__ FShared fcarve(uint8_t* raw) {
   s.tmem_base = reinterpret_cast<uint32_t*>(base + C::kMiscOff);
   s.abort_flag = reinterpret_cast<volatile int*>(base + C::kMiscOff + 4);
   return s;
+}
+
+// Element index (in bf16 units) of (row r, column kk < 16) in a K-major block
+// of 16 columns without swizzle: 8-row x 8-column core matrices of 128 bytes,
+// the two column halves 128 bytes apart, 8-row groups 256 bytes apart.
+__device__ __forceinline__ int nl_elem(int r, int kk) {
+  return ((r >> 3) * 256 + (kk >> 3) * 128 + (r & 7) * 16 + (kk & 7) * 2) >> 1;
+}
+
+__device__ __forceinline__ uint16_t bf16_bits_rn(float x) {
+  return __bfloat16_as_ushort(__float2bfloat16_rn(x));
+}
+
+__device__ __forceinline__ float bf16_value(uint16_t b) {
+  return __uint_as_float(static_cast<uint32_t>(b) << 16);
 }
 
 __device__ __forceinline__ int ld_acquire_gpu(const int32_t* p) {
@@ -910,8 +934,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t* dst = reinterpret_cast<uint32_t*>(sh.q + hf * C::kQHalfBytes + a.nrows * 128);
       for (int i = threadIdx.x; i < words; i += kThreads) dst[i] = 0u;
     }
-    fence_proxy_async_smem();
   }
+  // Operands of the extra pass-2 k-step, which adds each row's normaliser to
+  // its logits in the accumulator: keys x [1, 1, 1, 0 ...] against rows x
+  // [three bf16 parts of -lse2_j / c1, 0 ...] (the parts are written per item).
+  for (int i = threadIdx.x; i < kTileKeys * 16; i += kThreads) {
+    const int r = i >> 4, kk = i & 15;
+    reinterpret_cast<uint16_t*>(sh.ones)[nl_elem(r, kk)] = kk < 3 ? 0x3F80u : 0u;
+  }
+  for (int i = threadIdx.x; i < kRowsMax * 8; i += kThreads) reinterpret_cast<uint32_t*>(sh.nlb)[i] = 0u;
+  fence_proxy_async_smem();
   if (warp == kMmaWarp) {
     tmem_alloc(sh.tmem_base, kTmemCols);
     tmem_relinquish();
@@ -986,14 +1018,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------------ MMA
     if (lane == 0) {
       int kuse = 0, quse = 0, pair = 0;
+      int lpop = 0;                                // items whose normalisers the epilogue forms
       bool ok = true;
+      const uint64_t ones_desc = sdesc_kmajor_noswizzle(smem_u32(sh.ones), 128, 256);
+      const uint64_t nl_desc = sdesc_kmajor_noswizzle(smem_u32(sh.nlb), 128, 256);
+      const uint32_t idesc_nl = idesc_bf16_f32(128, a.nrows_pad);
       for (int item = blockIdx.x; item < fa.n_items && ok; item += gridDim.x) {
         const FItem it = fused_item(a, item);
         const int kt0 = it.kt0, kt1 = it.kt1;
-        if (kt1 == kt0) continue;
+        if (kt1 == kt0) {
+          if (a.mode != kModeH2O) ++lpop;          // (the epilogue still forms them)
+          continue;
+        }
         if (!mbar_wait(sh.q_full, quse & 1, sh.abort_flag, a.status)) break;
         ++quse;
         const uint32_t qbase = smem_u32(sh.q);
+        bool nl_ready = false;
         for (int pass = fa.single; pass < 2 && ok; ++pass)
           for (int kt = kt0; kt < kt1; ++kt) {
             const int kslot = kuse % C::SK;
@@ -1005,16 +1045,27 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tc_fence_after();
             const uint32_t kbase = smem_u32(sh.k + kslot * C::kKTileBytes);
-            if (pass == 0)
+            if (pass == 0) {
               issue_mma_rows_on_lanes<D>(qbase, kbase, tmem + ab * 256, nrt);
-            else
+            } else {
               issue_mma_keys_on_lanes<D>(qbase, kbase, tmem + ab * 256, a.nrows_pad);
+              // add the rows' normalisers (once the epilogue has written them)
+              if (!nl_ready) {
+                if (!mbar_wait(sh.lse_ready, lpop & 1, sh.abort_flag, a.status)) {
+                  ok = false;
+                  break;
+                }
+                nl_ready = true;
+              }
+              mma_bf16_ss(tmem + ab * 256, ones_desc, nl_desc, idesc_nl, 1u);
+            }
             mma_commit(&sh.acc_full[ab]);
             mma_commit(&sh.k_empty[kslot]);
             ++kuse;
             ++pair;
           }
         if (ok) mma_commit(sh.q_empty);
+        ++lpop;
       }
       mma_commit(sh.drain);
       mbar_wait(sh.drain, 0, nullptr, nullptr);
@@ -1161,8 +1212,19 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if (s > 0.f) nl = -(m + log2f(s));
         }
-        sh.lse[j] = nl;
         sh.pos[j] = p;
+        // -lse2_j / c1 as the sum of three bf16 parts (exact to ~2^-24); a row
+        // without keys gets -1e30, whose exponential is 0
+        const float x = nl > -INFINITY ? nl / c1 : -1.0e30f;
+        const uint16_t h0 = bf16_bits_rn(x);
+        const float r1 = x - bf16_value(h0);
+        const uint16_t h1 = bf16_bits_rn(r1);
+        const uint16_t h2 = bf16_bits_rn(r1 - bf16_value(h1));
+        uint16_t* nlr = reinterpret_cast<uint16_t*>(sh.nlb);
+        nlr[nl_elem(j, 0)] = h0;
+        nlr[nl_elem(j, 1)] = h1;
+        nlr[nl_elem(j, 2)] = h2;
+        fence_proxy_async_smem();
       }
       mbar_arrive(sh.lse_ready);
       ok = __all_sync(0xffffffffu, mbar_wait(sh.lse_ready, ipop & 1, sh.abort_flag, a.status));
@@ -1189,18 +1251,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_before();
             mbar_arrive(&sh.acc_empty[ab]);
           }
-          const float* nlp = sh.lse + j0 + h * 32;
+          // the accumulator holds S_jt - lse2_j / c1: the normaliser came in
+          // through the extra k-step, so no per-row value is loaded here
           if (fast) {
             float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
                              make_float2(0.f, 0.f)};
 #pragma unroll
             for (int i = 0; i < 32; i += 8) {
-              const float4 L0 = *reinterpret_cast<const float4*>(nlp + i);
-              const float4 L1 = *reinterpret_cast<const float4*>(nlp + i + 4);
-              acc[0] = __fadd2_rn(acc[0], exp2x2(__ffma2_rn(bits2(r, i), cc, make_float2(L0.x, L0.y))));
-              acc[1] = __fadd2_rn(acc[1], exp2x2(__ffma2_rn(bits2(r, i + 2), cc, make_float2(L0.z, L0.w))));
-              acc[2] = __fadd2_rn(acc[2], exp2x2(__ffma2_rn(bits2(r, i + 4), cc, make_float2(L1.x, L1.y))));
-              acc[3] = __fadd2_rn(acc[3], exp2x2(__ffma2_rn(bits2(r, i + 6), cc, make_float2(L1.z, L1.w))));
+#pragma unroll
+              for (int k = 0; k < 4; ++k)
+                acc[k] = __fadd2_rn(acc[k], exp2x2(__fmul2_rn(bits2(r, i + 2 * k), cc)));
             }
             const float2 s2 = __fadd2_rn(__fadd2_rn(acc[0], acc[1]), __fadd2_rn(acc[2], acc[3]));
             colsum += s2.x + s2.y;
@@ -1209,7 +1269,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             float s = 0.f;
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
-              const float e = fast_exp2(fmaf(__uint_as_float(r[i]), c1, nlp[i]));
+              const float e = fast_exp2(__uint_as_float(r[i]) * c1);
               s += (t <= pp[i]) ? e : 0.f;
             }
             colsum += s;

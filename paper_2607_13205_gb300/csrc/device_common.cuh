@@ -149,6 +149,18 @@ __device__ __forceinline__ uint64_t sdesc_kmajor_sw128(uint32_t saddr) {
   return d;
 }
 
+// Shared-memory matrix descriptor of a K-major bf16 operand without swizzle:
+// 8-row x 16-byte core matrices, `lbo` bytes apart along K and `sbo` bytes
+// apart between 8-row groups.
+__device__ __forceinline__ uint64_t sdesc_kmajor_noswizzle(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);   // start address
+  d |= static_cast<uint64_t>(lbo >> 4) << 16;             // leading (K) byte offset
+  d |= static_cast<uint64_t>(sbo >> 4) << 32;             // stride (M/N) byte offset
+  d |= static_cast<uint64_t>(1) << 46;                    // descriptor version
+  return d;                                               // layout type 0: no swizzle
+}
+
 // Instruction descriptor: kind::f16 with bf16 A and B (both K-major) and an
 // fp32 accumulator, shape M x N.
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {

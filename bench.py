@@ -480,11 +480,14 @@ def run_decode(args, batch, w, B, K, V, keep, k_out, v_out, stream, world, peaks
 def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_out, v_out, status,
             stream, world, seq_tokens):
     """The same step through the public calls with host buffers: the step's
-    inputs are copied from pinned host memory and the kept indices and the
-    compressed K/V read back, inside the timed region.  The step runs layer
-    slice by layer slice on three streams, so that a slice's host-to-device
-    copy, another slice's kernels and a third slice's read-back overlap (as
-    a prefill that hands its cache over layer by layer would)."""
+    inputs come from pinned host memory and the kept indices and the
+    compressed K/V are read back, inside the timed region.  K, the window
+    queries and the roles are copied to the device (the score reads all of
+    K); V stays in pinned host memory and kv_compact reads only its kept rows
+    over the host link.  The step runs layer slice by layer slice on three
+    streams, so that a slice's host-to-device copy, another slice's kernels
+    and a third slice's read-back overlap (as a prefill that hands its cache
+    over layer by layer would)."""
     import torch
 
     from paper_2607_13205_gb300 import rolekv as R
@@ -503,7 +506,6 @@ def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_o
     o_k = torch.empty(k_out.shape, dtype=k_out.dtype, pin_memory=True)
     o_v = torch.empty(v_out.shape, dtype=v_out.dtype, pin_memory=True)
     torch.cuda.synchronize()
-    bi = sum(t.numel() * t.element_size() for t in (h_qw, h_k, h_v, h_roles))
     bo = sum(t.numel() * t.element_size() for t in (o_keep, o_k, o_v))
 
     # layer slices; every tensor of the path has the layer axis first
@@ -536,7 +538,7 @@ def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_o
                            stream=stream)
         R.role_alloc_select(sb, scores[l0:l1], roles, params, keep[l0:l1], pool_k=pool_k, status=status,
                             stream=stream)
-        R.kv_compact(sb, K[l0:l1], V[l0:l1], keep[l0:l1], B, k_out[l0:l1], v_out[l0:l1], status=status,
+        R.kv_compact(sb, K[l0:l1], h_v[l0:l1], keep[l0:l1], B, k_out[l0:l1], v_out[l0:l1], status=status,
                      stream=stream)
 
     def e2e_step():
@@ -548,7 +550,6 @@ def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_o
                 s_in.wait_event(ev_done[i])            # the slice's last use by the kernels
                 qw[l0:l1].copy_(h_qw[l0:l1], non_blocking=True)
                 K[l0:l1].copy_(h_k[l0:l1], non_blocking=True)
-                V[l0:l1].copy_(h_v[l0:l1], non_blocking=True)
                 ev_in[i].record(s_in)
         stream.wait_event(ev_roles)
         for i in range(S):
@@ -566,6 +567,10 @@ def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_o
 
     e2e_step()
     torch.cuda.synchronize()
+    # bytes in per step: the copies plus the kept V rows the compaction reads
+    # from host memory (the step is the same every time)
+    v_rows = int((keep >= 0).sum().item())
+    bi = sum(t.numel() * t.element_size() for t in (h_qw, h_k, h_roles)) + v_rows * w.d * V.element_size()
     steps = max(1, min(args.steps, args.e2e_steps))
     barrier(world)
     torch.cuda.synchronize()
@@ -578,7 +583,8 @@ def run_e2e(args, score, batch, params, w, B, qw, K, V, roles, scores, keep, k_o
     dt = max_over_ranks(dt, world)
     return {"value": world * seq_tokens * steps / dt, "unit": UNIT, "h2d_bytes_per_step": bi,
             "d2h_bytes_per_step": bo, "steps": steps, "ms_per_step": dt / steps * 1e3,
-            "slices": S, "overlap": "layer slices: copy in, kernels and read-back on three streams"}
+            "slices": S, "overlap": "layer slices: copy in (K, queries, roles), kernels (the compaction "
+                                    "gathers the kept V rows from pinned host memory) and read-back on three streams"}
 
 
 # ------------------------------------------------------ CPU oracle baseline --

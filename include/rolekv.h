@@ -296,7 +296,9 @@ int role_alloc_select(const rolekv_batch* batch, const float* scores, const uint
  * every kept slot j; slots holding -1 become zero rows.  k_out / v_out are
  * dense bf16 [L][b][Hkv][K][d] (varlen: [L][Hkv][Ktot][d]) with the kept-index
  * layout of `budget` and the batch's kept_extra.  d must be a multiple of 8,
- * at most 256. */
+ * at most 256.  k and v may also point into pinned (page-locked, device-
+ * mapped) host memory: the kernel then reads only the kept rows across the
+ * host link, which moves B of the cache instead of all of it. */
 int kv_compact(const rolekv_batch* batch, rolekv_tensor k, rolekv_tensor v,
                const int32_t* keep_idx, float budget, void* k_out, void* v_out,
                int32_t* status_dev, void* stream);

@@ -559,6 +559,43 @@ def test_kv_compact_bit_exact(varlen):
         assert np.array_equal(kr[ok].astype(np.int32), ref_t.numpy())
 
 
+def test_kv_compact_reads_pinned_host_values():
+    """V left in pinned host memory: the compaction gathers the kept rows
+    across the host link and writes exactly what it writes from device V."""
+    w = _w("ragged", L=2, b=3, Hq=8, Hkv=2, n=900, seqlens=(900, 0, 333))
+    B = 0.2
+    roles = I.workload_roles(w, 5)
+    K, V = I.make_kv(w, roles, 5, device=DEV)
+    batch = lib_batch(w, DEV)
+    ob = oracle_batch(w)
+    rng = np.random.default_rng(12)
+    keep_np = np.full(batch.kept_shape(B), -1, dtype=np.int32)
+    cu_kept = ob.kept_offsets(B)
+    for u in range(ob.n_units):
+        l, s, h = ob.unit(u)
+        n, k = ob.seqlens[s], int(cu_kept[s + 1] - cu_kept[s])
+        if k:
+            keep_np[l, h, cu_kept[s]:cu_kept[s] + k - 1] = np.sort(rng.choice(n, size=k - 1, replace=False))
+    keep = torch.as_tensor(keep_np, device=DEV)
+    h_v = torch.empty(V.shape, dtype=V.dtype, pin_memory=True)
+    h_v.copy_(V)
+    outs = []
+    for vv in (V, h_v):
+        k_out = torch.full(R.compact_shape(batch, B), 3.0, dtype=torch.bfloat16, device=DEV)
+        v_out = torch.full_like(k_out, 3.0)
+        status = torch.zeros(1, dtype=torch.int32, device=DEV)
+        R.kv_compact(batch, K, vv, keep, B, k_out, v_out, status=status)
+        torch.cuda.synchronize()
+        assert int(status.item()) == 0
+        outs.append((k_out, v_out))
+    assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
+    vb, vo = I.bf16_bits(V), I.bf16_bits(outs[1][1])
+    for u in range(ob.n_units):
+        l, s, h = ob.unit(u)
+        sl = slice(cu_kept[s], cu_kept[s + 1])
+        assert np.array_equal(vo[l, h, sl], O.compact_unit(ob.kv_rows(vb, u), keep_np[l, h, sl]))
+
+
 # ------------------------------------------------------------- whole pipeline
 
 @pytest.mark.parametrize("name", ["tiny", "ragged_small", "ragged_small_ceil"])

@@ -1022,7 +1022,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       const uint64_t ones_desc = sdesc_kmajor_noswizzle(smem_u32(sh.ones), 128, 256);
       const uint64_t nl_desc = sdesc_kmajor_noswizzle(smem_u32(sh.nlb), 128, 256);
-      const uint32_t idesc_nl = idesc_bf16_f32(128, a.nrows_pad);
+      // pass 2 spans only the rows that exist, rounded up to 32 (224 of 256 at G = 7)
+      const int p2n = a.nrows_pad == 256 ? ((a.nrows + 31) & ~31) : a.nrows_pad;
+      const uint32_t idesc_nl = idesc_bf16_f32(128, p2n);
       for (int item = blockIdx.x; item < fa.n_items && ok; item += gridDim.x) {
         const FItem it = fused_item(a, item);
         const int kt0 = it.kt0, kt1 = it.kt1;
@@ -1048,7 +1050,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (pass == 0) {
               issue_mma_rows_on_lanes<D>(qbase, kbase, tmem + ab * 256, nrt);
             } else {
-              issue_mma_keys_on_lanes<D>(qbase, kbase, tmem + ab * 256, a.nrows_pad);
+              issue_mma_keys_on_lanes<D>(qbase, kbase, tmem + ab * 256, p2n);
               // add the rows' normalisers (once the epilogue has written them)
               if (!nl_ready) {
                 if (!mbar_wait(sh.lse_ready, lpop & 1, sh.abort_flag, a.status)) {
@@ -1094,8 +1096,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int nsub = kParts / nrt;
     // pass 2 mapping: one key lane, half of the rows of each owned tile
     const int kl = qd * 32 + lane;
-    const int p2cols = a.nrows_pad / 2;
-    const int j0 = gp * p2cols;
+    // (with two row tiles the second part takes the rows past 128 that exist,
+    // rounded up to 32, as pass 2's MMA computes only those)
+    const int p2cols = a.nrows_pad == 128 ? 64 : (gp == 0 ? 128 : ((a.nrows + 31) & ~31) - 128);
+    const int j0 = a.nrows_pad == 128 ? gp * 64 : gp * 128;
     const float c1 = a.c1;
     const float2 cc = make_float2(c1, c1);
     int pair = 0, xchg = 0;

@@ -59,6 +59,38 @@ def test_snapkv_score_matches_oracle(case):
             assert abs(ob.score_view(gpre, u).astype(np.float64).sum() - min(w.W, n) * w.G) < 1e-3 * min(w.W, n) * w.G
 
 
+@pytest.mark.parametrize("scale", [0.004, 0.5])
+@pytest.mark.parametrize("case", ["two_row_tiles_w64_multichunk", "varlen_g7"])
+def test_snapkv_and_h2o_with_explicit_scale(case, scale):
+    """A softmax scale other than 1/sqrt(d), from nearly flat (0.004) to
+    sharply peaked (0.5): both score kernels against the oracle at that scale
+    (the row normalisers enter pass 2 divided by scale * log2 e)."""
+    w = SNAPKV_CASES[case]
+    roles, K, V, qw = _snapkv_inputs(w, seed=4)
+    batch = lib_batch(w, DEV)
+    ob = oracle_batch(w)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    pre = torch.full(batch.score_shape(), -1.0, dtype=torch.float32, device=DEV)
+    R.snapkv_score(batch, qw, K, w.W, 1, pre, scale=scale, status=status)
+    ww = w if w.n <= 2100 else w.scaled(n=2100)
+    Kh = K if ww is w else K[:, :, :, :ww.n].contiguous()
+    bh = batch if ww is w else lib_batch(ww, DEV)
+    obh = ob if ww is w else oracle_batch(ww)
+    Q = I.make_q_full(ww, 4, device=DEV)
+    hs = torch.full(bh.score_shape(), -1.0, dtype=torch.float32, device=DEV)
+    R.h2o_score(bh, Q, Kh, hs, scale=scale, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    ref = O.snapkv_batch(ob, I.bf16_bits(qw), I.bf16_bits(K), w.W, 1, scale=scale)
+    got = pre.cpu().numpy()
+    for u, (rpre, _) in ref.items():
+        assert_scores_close(ob.score_view(got, u), rpre, f"{case} scale {scale} unit {u} snapkv")
+    href = O.h2o_batch(obh, I.bf16_bits(Q), I.bf16_bits(Kh), scale=scale)
+    hgot = hs.cpu().numpy()
+    for u, r in href.items():
+        assert_scores_close(obh.score_view(hgot, u), r, f"{case} scale {scale} unit {u} h2o")
+
+
 @pytest.mark.parametrize("case", ["varlen_short_empty", "two_row_tiles_w64_multichunk"])
 def test_snapkv_with_supplied_lse(case):
     """Single pass with the window rows' normalisers given (natural log)."""

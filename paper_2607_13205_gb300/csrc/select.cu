@@ -170,6 +170,8 @@ __device__ __forceinline__ void pass1(const UnitView& v, int n_roles, uint32_t b
   const uint32_t bmask = (1u << nb) - 1u;
   const int words_per_role = 1 << (nb - 1);
   for (int g = threadIdx.x; g < v.ngroups; g += NT) {
+    // the role bytes are loaded with the scores, not after the pooling
+    const uint32_t rw = load_roles(v.rp, v.off, v.n, g, v.rvec);
     float x[4 * (2 * NB + 1)];
 #pragma unroll
     for (int o = -NB; o <= NB; ++o) {
@@ -196,7 +198,6 @@ __device__ __forceinline__ void pass1(const UnitView& v, int n_roles, uint32_t b
       k[j] = ordered_key(m);
     }
     keys4[g] = make_uint4(k[0], k[1], k[2], k[3]);
-    const uint32_t rw = load_roles(v.rp, v.off, v.n, g, v.rvec);
     const uint32_t fb = floor_bits(4 * g - v.off, v.nf, v.n);
 #pragma unroll
     for (int j = 0; j < 4; ++j) {

@@ -733,8 +733,7 @@ struct FCfg {
   static constexpr int SK = 4;
   static constexpr int kQOff = 0;
   static constexpr int kKOff = kQOff + kQSlotBytes;
-  static constexpr int kLseOff = kKOff + SK * kKTileBytes;
-  static constexpr int kPosOff = kLseOff + kRowsMax * 4;
+  static constexpr int kPosOff = kKOff + SK * kKTileBytes;
   static constexpr int kRedOff = kPosOff + kRowsMax * 4;
   static constexpr int kMergeOff = kRedOff + (kParts - 1) * kTileKeys * 4;
   // the extra pass-2 k-step: row normalisers (256 rows) against ones (128
@@ -755,7 +754,6 @@ struct FShared {
   uint8_t* k;
   uint8_t* nlb;      // [256 rows][16] bf16: -lse2_j / c1 in three parts, then zeros
   uint8_t* ones;     // [128 keys][16] bf16: 1, 1, 1, then zeros
-  float* lse;        // negated log2 normalisers of the current item's rows
   int32_t* pos;
   float* red;
   float2* merge;
@@ -774,7 +772,6 @@ __device__ __forceinline__ FShared fcarve(uint8_t* raw) {
   FShared s;
   s.q = base + C::kQOff;
   s.k = base + C::kKOff;
-  s.lse = reinterpret_cast<float*>(base + C::kLseOff);
   s.pos = reinterpret_cast<int32_t*>(base + C::kPosOff);
   s.red = reinterpret_cast<float*>(base + C::kRedOff);
   s.merge = reinterpret_cast<float2*>(base + C::kMergeOff);

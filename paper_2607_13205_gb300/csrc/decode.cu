@@ -194,10 +194,24 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const Decod
     const float c1 = a.c1;
     const int d0 = lane * DPL;
     float* pw = &pbuf[warp][0][0];
+    // kept-index words of this lane's two rows, loaded one stage ahead so that
+    // their latency hides behind the stage before
+    auto load_idx = [&](int stt, int32_t& ia, int32_t& ib) {
+      const int trr = r0 + stt * kStageRows + warp * kTileRows;
+      ia = (idx != nullptr && trr + g < r1) ? __ldg(idx + trr + g) : 0;
+      ib = (idx != nullptr && trr + g + 8 < r1) ? __ldg(idx + trr + g + 8) : 0;
+    };
+    int32_t ia_cur, ib_cur;
+    load_idx(0, ia_cur, ib_cur);
     for (int st = 0; st < nst; ++st) {
       const int slot = st % kStages;
+      int32_t ia_next = 0, ib_next = 0;
+      if (st + 1 < nst) load_idx(st + 1, ia_next, ib_next);
       const bool got = mbar_wait(&full_bar[slot], (st / kStages) & 1, &abort_flag, a.status);
       if (!__all_sync(0xffffffffu, got)) break;
+      const int32_t ia = ia_cur, ib = ib_cur;
+      ia_cur = ia_next;
+      ib_cur = ib_next;
       const int tr0 = r0 + st * kStageRows + warp * kTileRows;   // first row of this warp's tile
       const uint8_t* kt = ks + slot * kStageRows * KSTR + warp * kTileRows * KSTR;
       const uint8_t* vt = vs + slot * kStageRows * VSTR + warp * kTileRows * VSTR;
@@ -210,8 +224,8 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const Decod
                    lds32(ka + 8 * KSTR + 32 * k + 16), qb[k][0], qb[k][1]);
         // rows g and g + 8: inside the split, and a kept slot
         const int ra = tr0 + g, rb = tr0 + g + 8;
-        const bool oka = ra < r1 && (idx == nullptr || __ldg(idx + ra) >= 0);
-        const bool okb = rb < r1 && (idx == nullptr || __ldg(idx + rb) >= 0);
+        const bool oka = ra < r1 && (idx == nullptr || ia >= 0);
+        const bool okb = rb < r1 && (idx == nullptr || ib >= 0);
         const float s0 = oka ? c[0] * c1 : -INFINITY, s1 = oka ? c[1] * c1 : -INFINITY;
         const float s2 = okb ? c[2] * c1 : -INFINITY, s3 = okb ? c[3] * c1 : -INFINITY;
         float tm0 = fmaxf(s0, s2), tm1 = fmaxf(s1, s3);

@@ -30,6 +30,7 @@
 
 #include <cmath>
 #include <cstdint>
+#include <type_traits>
 
 #include "device_common.cuh"
 #include "internal.h"
@@ -1245,37 +1246,46 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!ok) break;
         tc_fence_after();
         float colsum = 0.f;
-        uint32_t r[32];
-        for (int h = 0; h < p2cols / 32; ++h) {
-          tmem_load_cols<32>(tmem + lane_base + ab * 256 + j0 + h * 32, r);
-          if (h + 1 == p2cols / 32) {
-            tc_fence_before();
-            mbar_arrive(&sh.acc_empty[ab]);
-          }
-          // the accumulator holds S_jt - lse2_j / c1: the normaliser came in
-          // through the extra k-step, so no per-row value is loaded here
-          if (fast) {
-            float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
-                             make_float2(0.f, 0.f)};
-#pragma unroll
-            for (int i = 0; i < 32; i += 8) {
-#pragma unroll
-              for (int k = 0; k < 4; ++k)
-                acc[k] = __fadd2_rn(acc[k], exp2x2(__fmul2_rn(bits2(r, i + 2 * k), cc)));
+        // drain the owned columns NC at a time (64 when they divide: two
+        // loads in flight per wait, and the buffer released halfway)
+        auto drain = [&](auto nc_tag) {
+          constexpr int NC = decltype(nc_tag)::value;
+          uint32_t r[NC];
+          for (int h = 0; h < p2cols / NC; ++h) {
+            tmem_load_cols<NC>(tmem + lane_base + ab * 256 + j0 + h * NC, r);
+            if (h + 1 == p2cols / NC) {
+              tc_fence_before();
+              mbar_arrive(&sh.acc_empty[ab]);
             }
-            const float2 s2 = __fadd2_rn(__fadd2_rn(acc[0], acc[1]), __fadd2_rn(acc[2], acc[3]));
-            colsum += s2.x + s2.y;
-          } else {
-            const int32_t* pp = sh.pos + j0 + h * 32;
-            float s = 0.f;
+            // the accumulator holds S_jt - lse2_j / c1: the normaliser came in
+            // through the extra k-step, so no per-row value is loaded here
+            if (fast) {
+              float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                               make_float2(0.f, 0.f)};
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const float e = fast_exp2(__uint_as_float(r[i]) * c1);
-              s += (t <= pp[i]) ? e : 0.f;
+              for (int i = 0; i < NC; i += 8) {
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+                  acc[k] = __fadd2_rn(acc[k], exp2x2(__fmul2_rn(bits2(r, i + 2 * k), cc)));
+              }
+              const float2 s2 = __fadd2_rn(__fadd2_rn(acc[0], acc[1]), __fadd2_rn(acc[2], acc[3]));
+              colsum += s2.x + s2.y;
+            } else {
+              const int32_t* pp = sh.pos + j0 + h * NC;
+              float s = 0.f;
+#pragma unroll
+              for (int i = 0; i < NC; ++i) {
+                const float e = fast_exp2(__uint_as_float(r[i]) * c1);
+                s += (t <= pp[i]) ? e : 0.f;
+              }
+              colsum += s;
             }
-            colsum += s;
           }
-        }
+        };
+        if (p2cols % 64 == 0)
+          drain(std::integral_constant<int, 64>{});
+        else
+          drain(std::integral_constant<int, 32>{});
         // add the group's two row halves of this key and write s(t)
         if (gp != 0) {
           ok = mbar_wait(&sh.red_empty[grp], (xchg & 1) ^ 1, sh.abort_flag, a.status);

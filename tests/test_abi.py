@@ -145,3 +145,33 @@ def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
     monkeypatch.setattr(R, "_lib", None)
     with pytest.raises(RuntimeError, match="missing"):
         R.kept_count(10, 0.5)
+
+def test_struct_layouts_match_the_header(tmp_path):
+    """The binding's ctypes structs have the sizes and field offsets that a C
+    compiler gives the header's structs (the header also compiles as C99)."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    fields = {"rolekv_batch": [f for f, _ in R.BatchDesc._fields_],
+              "rolekv_select_params": [f for f, _ in R.SelectParams._fields_],
+              "rolekv_tensor": [f for f, _ in R.Tensor._fields_]}
+    lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "rolekv.h"', "int main(void) {"]
+    for st, fs in fields.items():
+        lines.append(f'  printf("{st} size %zu\\n", sizeof({st}));')
+        for f in fs:
+            lines.append(f'  printf("{st} {f} %zu\\n", offsetof({st}, {f}));')
+    lines += ["  return 0;", "}"]
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "layout"
+    subprocess.run([cc, "-std=c99", "-Wall", "-Werror", "-I", inc, str(src), "-o", str(exe)], check=True)
+    out = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split("\n")
+    got = {tuple(l.split()[:-1]): int(l.split()[-1]) for l in out if l}
+    for st, cls in (("rolekv_batch", R.BatchDesc), ("rolekv_select_params", R.SelectParams),
+                    ("rolekv_tensor", R.Tensor)):
+        assert got[(st, "size")] == ctypes.sizeof(cls), st
+        for f in fields[st]:
+            assert got[(st, f)] == getattr(cls, f).offset, (st, f)

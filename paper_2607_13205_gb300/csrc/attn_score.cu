@@ -11,7 +11,10 @@
 //     epilogue thread owns a row and keeps its running max and sum of exp2.
 //   pass 2 (colsum):   S^T = K Q^T with keys on the TMEM lanes; each epilogue
 //     thread owns a key and sums exp2(S c - lse2_j) over the rows
-//     thread-locally, so no cross-thread reduction is needed.
+//     thread-locally, so no cross-thread reduction is needed.  In the
+//     persistent kernel the normalisers enter the accumulator through a ninth
+//     MMA k-step (keys x ones against rows x -lse2_j / c1), so the epilogue
+//     loads no per-row value from shared memory.
 //
 // In both passes one producer warp streams 128-key K tiles and 256-row query
 // blocks into 128-byte-swizzled shared memory with TMA, one warp issues
@@ -938,7 +941,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // [three bf16 parts of -lse2_j / c1, 0 ...] (the parts are written per item).
   for (int i = threadIdx.x; i < kTileKeys * 16; i += kThreads) {
     const int r = i >> 4, kk = i & 15;
-    reinterpret_cast<uint16_t*>(sh.ones)[nl_elem(r, kk)] = kk < 3 ? 0x3F80u : 0u;
+    reinterpret_cast<uint16_t*>(sh.ones)[nl_elem(r, kk)] = kk < 3 ? 0x3F80u : 0u;   // bf16 1.0
   }
   for (int i = threadIdx.x; i < kRowsMax * 8; i += kThreads) reinterpret_cast<uint32_t*>(sh.nlb)[i] = 0u;
   fence_proxy_async_smem();

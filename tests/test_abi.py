@@ -118,6 +118,11 @@ def test_host_rejects_bad_arguments(lib):
     narrow.kept_extra = 1
     rc = lib.role_alloc_select(ctypes.byref(narrow), f, f, ctypes.byref(p_ceil), 1, f, None, None, None, None)
     assert rc == R.ERR_INVALID_ARG and b"kept_extra >= 2" in lib.rolekv_last_error()
+    # the one-call path applies the same check before it launches anything
+    rc = lib.rolekv_compress(ctypes.byref(narrow), R.Tensor(256, 0, 32 * 128, 8 * 128, 128),
+                             R.Tensor(256, 2 * 1000 * 128, 1000 * 128, 0, 128), t, 32, 7, 0.0, None, f,
+                             ctypes.byref(p_ceil), f, f, f, None, f, 1 << 30, None, None)
+    assert rc == R.ERR_INVALID_ARG and b"kept_extra" in lib.rolekv_last_error()
     neg = _batch()
     neg.kept_extra = -1
     rc = lib.kv_compact(ctypes.byref(neg), t, t, f, 0.1, f, f, None, None)

@@ -567,6 +567,14 @@ def pin_quest_bound(O, rng):
     short = rng.standard_normal((3, d))
     qbar3 = qw[:, :3].reshape(-1, d).mean(axis=0)
     assert np.allclose(O.quest_score(qw, short, W, 1), short @ qbar3, rtol=1e-12, atol=1e-12)
+    # hand-worked pages where the per-dimension bound lies strictly above the
+    # page's best dot product (so an exact per-page maximum would fail here)
+    g = _golden("quest_bound_worked_examples.json")
+    qg = np.asarray(g["q_win"], dtype=np.float64)
+    for case in g["cases"]:
+        keys = np.asarray(case["keys"], dtype=np.float64)
+        got = O.quest_score(qg, keys, g["W"], case["page"])
+        assert np.array_equal(got, np.asarray(case["bound"], dtype=np.float64)), (case, got)
 
 
 def pin_decode_attention(O, rng):
@@ -595,6 +603,19 @@ def pin_decode_attention(O, rng):
     flags = np.concatenate([ok, np.zeros(5, dtype=bool)])
     assert np.allclose(O.decode_attention(q, junk_k, junk_v, flags, 0.5), o, rtol=1e-12, atol=1e-12)
     assert np.all(O.decode_attention(q, k, v, np.zeros(m, dtype=bool), 0.5) == 0)
+    # closed form at a scale other than 1: two keys 4 e_0 ("hot") and two zero
+    # keys, values 8 e_j.  With scale 1/4 a query (ln 3, ...) gives the hot
+    # keys logit ln 3 and the cold ones 0, so the weights are 3/8, 3/8, 1/8,
+    # 1/8 and the output (3, 3, 1, 1); a query (-ln 3, ...) gives weights
+    # 1/8, 1/8, 3/8, 3/8 and the output (1, 1, 3, 3).  Components of q along
+    # dimensions where every key is 0 do not matter.
+    ln3 = math.log(3.0)
+    qs = np.array([[ln3, 0.0, 0.0, 0.0], [-ln3, 0.7, -1.1, 0.3]])
+    ks = np.array([[4.0, 0, 0, 0], [4.0, 0, 0, 0], [0.0, 0, 0, 0], [0.0, 0, 0, 0]])
+    vs = 8.0 * np.eye(4)
+    want = np.array([[3.0, 3.0, 1.0, 1.0], [1.0, 1.0, 3.0, 3.0]])
+    got = O.decode_attention(qs, ks, vs, np.ones(4, dtype=bool), 0.25)
+    assert np.allclose(got, want, rtol=0, atol=1e-12), got
 
 
 ALL_PINS = [

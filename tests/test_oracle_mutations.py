@@ -207,6 +207,21 @@ def _m_quest_window_start(O):
                  "q = np.asarray(q_win, dtype=np.float64)", ["quest_score"])
 
 
+def _m_quest_exact_page_max(O):
+    # the exact best dot product of the page: also an upper bound, exact for
+    # one-token pages and for equal keys, but not Quest's per-dimension bound
+    _from_source(O, "np.maximum(qbar * lo, qbar * hi).sum()", "(blk @ qbar).max()", ["quest_score"])
+
+
+def _m_decode_scale_squared(O):
+    _from_source(O, "logits = scale * (q @ kk.T)", "logits = scale * scale * (q @ kk.T)",
+                 ["decode_attention"])
+
+
+def _m_decode_no_scale(O):
+    _from_source(O, "logits = scale * (q @ kk.T)", "logits = (q @ kk.T)", ["decode_attention"])
+
+
 def _m_decode_keeps_padding(O):
     _from_source(O, "kk, vv = k[valid], v[valid]", "kk, vv = k, v", ["decode_attention"])
 
@@ -255,6 +270,7 @@ MUTATIONS = [
     _m_round_not_ceil, _m_no_redistribution, _m_renormalise_all_buckets, _m_remainder_ties_high,
     _m_ties_to_high_index, _m_interleaved_gqa, _m_compact_off_by_one, _m_fair_uses_alpha,
     _m_floor_outside_budget, _m_floor_counts_whole_row, _m_quest_max_only, _m_quest_window_start,
+    _m_quest_exact_page_max, _m_decode_scale_squared, _m_decode_no_scale,
     _m_decode_keeps_padding, _m_decode_unnormalised, _m_slack_from_all_roles, _m_slack_waterfills,
     _m_slack_not_filled, _m_ceil_floors, _m_ceil_no_waterfill, _m_ceil_unnormalised,
     _m_ceil_rows_not_widened,

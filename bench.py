@@ -136,20 +136,66 @@ class ClockSampler:
 
 # ------------------------------------------------------- algorithmic counts --
 
-# DRAM bytes (read + write) of one launch of the dominant kernel, from ncu's
-# dram__bytes_read.sum + dram__bytes_write.sum on the same kernel build.  The
-# long workload's fused score launch was captured on its first 2 layers
-# (64 units: 925.2 + 10.8 MB) and scaled by units (x16); any change to that
-# kernel makes this stale, and then it must be measured again.
-MEASURED_TRAFFIC = {("long", "snapkv", "score"): (925.2e6 + 10.8e6) * 16,
-                    ("long", "quest", "score"): (541.1e6 + 5.8e6) * 16}
+# DRAM bytes (read + write) of one launch of a kernel come from ncu's
+# dram__bytes_read.sum + dram__bytes_write.sum, captured on a smaller case of
+# the same workload and scaled by units (the kernels stream each unit's keys,
+# so their traffic grows in proportion).  profiles/dram_traffic.md holds the
+# captures, each with a hash of the kernel's source files at capture time; a
+# capture whose sources have changed since is stale and gives null.
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "dram_traffic.md")
+KERNEL_SOURCES = {
+    ("snapkv", "score"): ["attn_score.cu", "device_common.cuh", "internal.h"],
+    ("h2o", "score"): ["attn_score.cu", "device_common.cuh", "internal.h"],
+    ("quest", "score"): ["quest.cu", "internal.h"],
+    ("snapkv", "select"): ["select.cu", "internal.h"],
+    ("snapkv", "compact"): ["compact.cu", "internal.h"],
+}
+
+
+def source_hash(files) -> str:
+    import hashlib
+    h = hashlib.sha256()
+    for f in files:
+        with open(os.path.join(ROOT, "paper_2607_13205_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def measured_traffic(workload: str, score_kind: str, kernel: str, single: bool = False):
+    """(bytes per full launch, note) from profiles/dram_traffic.md, or (None,
+    reason).  Rows: | workload | score | kernel | pass | units captured |
+    units full | dram read MB | dram write MB | source hash |."""
+    srcs = KERNEL_SOURCES.get((score_kind, kernel)) or KERNEL_SOURCES.get(("snapkv", kernel))
+    if srcs is None or not os.path.exists(TRAFFIC_FILE):
+        return None, "no capture"
+    want = source_hash(srcs)
+    mode = "one" if single else "two"
+    with open(TRAFFIC_FILE) as f:
+        for line in f:
+            cells = [c.strip() for c in line.strip().strip("|").split("|")]
+            if len(cells) != 9 or cells[0] != workload or cells[1] != score_kind or cells[2] != kernel:
+                continue
+            if kernel == "score" and score_kind != "quest" and cells[3] != mode:
+                continue
+            try:
+                u_cap, u_full = float(cells[4]), float(cells[5])
+                rd, wr = float(cells[6]), float(cells[7])
+            except ValueError:
+                continue
+            if cells[8] != want:
+                return None, f"stale: captured on sources {cells[8]}, now {want}"
+            return (rd + wr) * 1e6 * u_full / u_cap, (f"ncu on {cells[4]} of {cells[5]} units, "
+                                                      f"scaled by units; sources {want}")
+    return None, "no capture for this workload"
 
 
 def path_counts(w, B, score_kind="snapkv"):
-    """Algorithmic bytes / flops per step of each kernel of the path: K read
-    once, the queries, the pre-pool score written and read once, the kept K/V
-    rows read and written, the kept index written and read.  Variable-length
-    batches use their mean length (exact for the sums of per-token terms)."""
+    """Algorithmic bytes / flops per step of each kernel of the path (the
+    method's own work: K read once, one Q K^T, the queries, the pre-pool score
+    written and read once, the kept K/V rows read and written, the kept index
+    written and read).  'hw_flops' is the contraction the exact two-pass
+    kernel actually runs (Q K^T twice).  Variable-length batches use their
+    mean length (exact for the sums of per-token terms)."""
     U = w.L * w.b * w.Hkv
     n = (sum(w.seqlens) / w.b) if w.varlen else w.n
     d = w.d
@@ -160,9 +206,8 @@ def path_counts(w, B, score_kind="snapkv"):
         qbytes = U * w.G * n * d * 2
         kbytes = U * n * d * 2
         return {
-            # one fused launch: both passes' QK^T, K and the queries read once,
-            # the scores written once
-            "score": {"bytes": kbytes + qbytes + U * n * 4, "flops": 2.0 * flops},
+            # K and the queries read once, the scores written once
+            "score": {"bytes": kbytes + qbytes + U * n * 4, "flops": flops, "hw_flops": 2.0 * flops},
             "select": {"bytes": U * n * 4 + w.b * n + U * K * 4, "flops": 0.0},
             "compact": {"bytes": U * K * 4 + 2 * 2 * U * K * d * 2, "flops": 0.0},
             "path_bytes": kbytes + qbytes + U * n * 8 + U * K * 8 + 2 * 2 * U * K * d * 2 + w.b * n,
@@ -176,13 +221,43 @@ def path_counts(w, B, score_kind="snapkv"):
         # one pass over K for the page bounds, no contraction
         flops = 0.0
     return {
-        # both passes in one kernel: K crosses HBM once, the QK^T is done twice
-        "score": {"bytes": kbytes + qbytes + U * n * 4, "flops": 2 * flops},
+        "score": {"bytes": kbytes + qbytes + U * n * 4, "flops": flops, "hw_flops": 2.0 * flops},
         "select": {"bytes": U * n * 4 + w.b * n + U * K * 4, "flops": 0.0},
         "compact": {"bytes": U * K * 4 + 2 * 2 * U * K * d * 2, "flops": 0.0},
         "path_bytes": kbytes + qbytes + U * n * 8 + U * K * 8 + 2 * 2 * U * K * d * 2 + w.b * n,
         "kept": K,
     }
+
+
+def roofline(counts, per_kernel, peaks, names, workload, score_kind, layers_override, traffic_arg):
+    """The dominant kernel's roofline: bound by its algorithmic bytes or
+    flops, whichever takes longer at the measured peaks; achieved = that work
+    / the kernel's mean launch time."""
+    dom = max(names, key=lambda k: per_kernel[k])
+    dk = counts[dom]
+    t_dom = per_kernel[dom] / 1e3
+    t_hbm = dk["bytes"] / (peaks["hbm_gbs"] * 1e9)
+    t_tc = dk["flops"] / (peaks["bf16_tflops"] * 1e12) if dk["flops"] else 0.0
+    if t_tc > t_hbm:
+        roof = {"bound": "tensor", "achieved": dk["flops"] / t_dom / 1e12,
+                "peak": peaks["bf16_tflops"], "unit": "TFLOP/s"}
+    else:
+        roof = {"bound": "hbm", "achieved": dk["bytes"] / t_dom / 1e9, "peak": peaks["hbm_gbs"],
+                "unit": "GB/s"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["kernel"] = dom
+    roof["algorithmic"] = {"bytes": dk["bytes"], "flops": dk["flops"]}
+    if dk.get("hw_flops"):
+        # the exact two-pass score runs Q K^T twice: tensor-pipe use of that work
+        roof["hw_tensor_frac"] = dk["hw_flops"] / t_dom / 1e12 / peaks["bf16_tflops"]
+    if traffic_arg is not None:
+        roof["traffic"], roof["traffic_note"] = traffic_arg, "given on the command line"
+    elif layers_override:
+        roof["traffic"], roof["traffic_note"] = None, "layer count overridden"
+    else:
+        roof["traffic"], roof["traffic_note"] = measured_traffic(workload, score_kind, dom)
+    roof["peak_source"] = peaks["source"] + " (burst)"
+    return roof
 
 
 # ----------------------------------------------------------------- GPU arm --
@@ -296,22 +371,8 @@ def run_gpu(args):
 
     peaks = load_peaks()
     counts = path_counts(w, B, args.score)
-    dom = max(names, key=lambda k: per_kernel[k])
-    dk = counts[dom]
-    t_dom = per_kernel[dom] / 1e3
-    t_hbm = dk["bytes"] / (peaks["hbm_gbs"] * 1e9)
-    t_tc = dk["flops"] / (peaks["bf16_tflops"] * 1e12) if dk["flops"] else 0.0
-    if t_tc > t_hbm:
-        roof = {"bound": "tensor", "achieved": dk["flops"] / t_dom / 1e12,
-                "peak": peaks["bf16_tflops"], "unit": "TFLOP/s"}
-    else:
-        roof = {"bound": "hbm", "achieved": dk["bytes"] / t_dom / 1e9, "peak": peaks["hbm_gbs"],
-                "unit": "GB/s"}
-    roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["kernel"] = dom
-    roof["traffic"] = (args.traffic if args.traffic is not None
-                       else (MEASURED_TRAFFIC.get((w.name, args.score, dom)) if not args.layers else None))
-    roof["peak_source"] = peaks["source"] + " (burst)"
+    roof = roofline(counts, per_kernel, peaks, names, w.name, "h2o" if h2o else args.score,
+                    args.layers, args.traffic)
     path_frac = counts["path_bytes"] / (ms_step / 1e3) / 1e9 / peaks["hbm_gbs"]
     tensor_util = {nm: counts[nm]["flops"] / (per_kernel[nm] / 1e3) / 1e12 / peaks["bf16_tflops"]
                    for nm in names if counts[nm]["flops"] > 0}
@@ -341,6 +402,10 @@ def run_gpu(args):
         result["single_pass"] = run_single_pass(args, batch, params, w, B, qw, K, V, roles, scores,
                                                 keep, k_out, v_out, ws, status, stream, world,
                                                 seq_tokens)
+    if h2o and not args.no_single_pass:
+        result["single_pass"] = run_h2o_single_pass(args, batch, params, w, B, qw, K, V, roles, scores,
+                                                    keep, k_out, v_out, ws, status, stream, world,
+                                                    seq_tokens, peaks, counts)
     if not h2o and not args.no_decode:
         result["decode"] = run_decode(args, batch, w, B, K, V, keep, k_out, v_out, stream, world, peaks)
     if not args.no_e2e:
@@ -431,6 +496,77 @@ def run_single_pass(args, batch, params, w, B, qw, K, V, roles, scores, keep, k_
     return {"value": world * seq_tokens * steps / (total / 1e3), "unit": UNIT,
             "ms_per_step": total / steps, "score_ms": score_ms, "steps": steps,
             "lse": "window normalisers supplied by the caller (computed once, untimed)"}
+
+
+def prefill_lse(w, Q, K):
+    """Natural-log softmax normaliser of every causal prefill query row, in
+    h2o_score's layout (dense [L][b][Hq][n]), as the prefill attention would
+    hand it over (computed here once, with fp32 torch matmuls, outside any
+    timed region)."""
+    import torch
+
+    L, b, G, n, d = w.L, w.b, w.G, w.n, w.d
+    lse = torch.empty((L, b, w.Hq, n), dtype=torch.float32, device=Q.device)
+    scale = 1.0 / math.sqrt(d)
+    above = torch.ones((n, n), dtype=torch.bool, device=Q.device).triu_(1)   # keys after the query
+    for l in range(L):
+        for s in range(b):
+            for h in range(w.Hkv):
+                k = K[l, s, h].float()
+                q = Q[l, s, h * G:(h + 1) * G].float()                 # [G][n][d]
+                logits = torch.matmul(q, k.T) * scale
+                logits.masked_fill_(above, float("-inf"))
+                lse[l, s, h * G:(h + 1) * G] = torch.logsumexp(logits, dim=-1)
+                del logits
+    return lse
+
+
+def run_h2o_single_pass(args, batch, params, w, B, Q, K, V, roles, scores, keep, k_out, v_out, ws,
+                        status, stream, world, seq_tokens, peaks, counts):
+    """The H2O step with every query row's normaliser supplied by the caller
+    (the prefill attention's softmax LSE): the score multiplies the keys once,
+    then selection and compaction."""
+    import torch
+
+    from paper_2607_13205_gb300 import rolekv as R
+
+    if w.varlen:
+        return None
+    torch.backends.cuda.matmul.allow_tf32 = False
+    lse = prefill_lse(w, Q, K)
+    torch.cuda.synchronize()
+
+    def score():
+        R.h2o_score(batch, Q, K, scores, lse=lse, ws=ws, status=status, stream=stream)
+
+    def rest():
+        R.role_alloc_select(batch, scores, roles, params, keep, pool_k=1, status=status, stream=stream)
+        R.kv_compact(batch, K, V, keep, B, k_out, v_out, status=status, stream=stream)
+
+    for _ in range(3):
+        score()
+        rest()
+    steps = max(1, args.steps)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2 * steps + 1)]
+    torch.cuda.synchronize()
+    barrier(world)
+    ev[0].record(stream)
+    for i in range(steps):
+        score()
+        ev[2 * i + 1].record(stream)
+        rest()
+        ev[2 * i + 2].record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    total = max_over_ranks(ev[0].elapsed_time(ev[-1]), world)
+    score_ms = sum(ev[2 * i].elapsed_time(ev[2 * i + 1]) for i in range(steps)) / steps
+    if int(status.item()) != 0:
+        raise SystemExit(f"device status {int(status.item())} in the single-pass H2O steps")
+    flops = counts["score"]["flops"]
+    return {"value": world * seq_tokens * steps / (total / 1e3), "unit": UNIT,
+            "ms_per_step": total / steps, "score_ms": score_ms, "steps": steps,
+            "score_tensor_frac": flops / (score_ms / 1e3) / 1e12 / peaks["bf16_tflops"],
+            "lse": "every query row's normaliser supplied by the caller (computed once, untimed)"}
 
 
 def run_decode(args, batch, w, B, K, V, keep, k_out, v_out, stream, world, peaks):
@@ -761,13 +897,45 @@ def main(argv=None):
                     help="override the layer count (smaller cases for profiling)")
     ap.add_argument("--traffic", type=float, default=None,
                     help="dram bytes per launch of the dominant kernel from an ncu capture")
+    ap.add_argument("--all-configs", action="store_true",
+                    help="one JSON line per benchmark configuration: tiny, llama8b at each of "
+                         "its budgets, long, h2o and ragged (no e2e or decode legs)")
     args = ap.parse_args(argv)
     if args.warmup < 3 and args.impl == "ours":
         print("warning: fewer than 3 warm-up steps", file=sys.stderr)
     if args.impl == "reference":
         run_reference(args)
+    elif args.all_configs:
+        run_all_configs(args)
     else:
         run_gpu(args)
+
+
+def run_all_configs(args):
+    """Every benchmark configuration in turn on one GPU (the budgets of the
+    8B configuration each), one JSON line each, with a shorter CPU sample."""
+    import gc
+
+    import torch
+
+    from paper_2607_13205_gb300 import inputs as I
+
+    _, world, _ = dist_env()
+    if world > 1:
+        raise SystemExit("--all-configs runs on one GPU")
+    sweep = [("tiny", B) for B in I.WORKLOADS["tiny"].budgets]
+    sweep += [("llama8b", B) for B in I.WORKLOADS["llama8b"].budgets]
+    sweep += [("long", B) for B in I.WORKLOADS["long"].budgets]
+    sweep += [("h2o", B) for B in I.WORKLOADS["h2o"].budgets]
+    sweep += [("ragged", B) for B in I.WORKLOADS["ragged"].budgets]
+    for name, B in sweep:
+        a = argparse.Namespace(**vars(args))
+        a.workload, a.budget = name, B
+        a.no_e2e, a.no_decode = True, True
+        a.cpu_seconds = min(args.cpu_seconds, 5.0)
+        run_gpu(a)
+        gc.collect()
+        torch.cuda.empty_cache()
 
 
 if __name__ == "__main__":

@@ -214,8 +214,13 @@ int snapkv_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k
  *   32768 tokens); with pool_k > 1, scores_prepool is required, because the
  *   pre-pool scores are an output here, not scratch.
  *   Set-up: the first call on each device looks up the array's device address
- *   (cudaGetSymbolAddress) with that device current and caches it; make that
- *   first call before any stream capture.
+ *   (cudaGetSymbolAddress) with that device current and caches it for the
+ *   rest of the process; make that first call before any stream capture.
+ *   The cached address belongs to the device's primary context (the one the
+ *   CUDA runtime uses by default): call this entry point only from that
+ *   context, and not after cudaDeviceReset on the device.
+ *   Empty batches (no tokens) return ROLEKV_OK without touching any buffer,
+ *   as snapkv_score does.
  *   Sharing: every call on a device uses the same array and leaves its
  *   contents behind; each call overwrites all it reads, so nothing needs
  *   clearing, but calls that overlap on the GPU (other streams, other host
@@ -269,13 +274,20 @@ int decode_attention(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k
  * of the KV head and every causal query position q >= t of p_t(q).
  *   q       bf16 prefill queries of every position: dense [L][b][Hq][n][d] or
  *           varlen [L][T][Hq][d], addressed by its strides.
+ *   scale   softmax scale; <= 0 selects 1/sqrt(d).
+ *   lse     optional fp32 natural-log softmax normaliser of every query row
+ *           over its causal keys (the softmax_lse a prefill attention already
+ *           produces): dense [L][b][Hq][n_max], varlen [L][Hq][T] (sequence s
+ *           at columns cu[s] .. cu[s+1]-1), 4-byte aligned.  Given, the keys
+ *           are read and multiplied once (pass 2 only); NULL: the normalisers
+ *           are computed here, in a first pass over the same key tiles.
  *   scores  fp32 score array.  No pooling (the H2O score has none).  Each
  *           score is a sum of per-query-block parts added atomically, in an
  *           order that varies between runs (about 1e-7 relative).
  * d must be 64 or 128 and G <= 8. */
 int h2o_score(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k, float scale,
-              float* scores, void* workspace, size_t workspace_bytes, int32_t* status_dev,
-              void* stream);
+              const float* lse, float* scores, void* workspace, size_t workspace_bytes,
+              int32_t* status_dev, void* stream);
 
 /* Role-conditional allocation and per-bucket top-k (Section 4.1, Algorithm 1).
  *   scores        fp32 score array (pooled SnapKV, H2O, or any score).
@@ -338,6 +350,19 @@ const char* rolekv_version(void);
  * It lets a caller check, without a fault, that a stuck wait is reported and
  * the context stays usable. */
 int rolekv_selftest_wait(int64_t limit_ns, int32_t* status_dev, void* stream);
+
+/* Diagnostic (no counterpart in the paper): arms the next two-pass SnapKV
+ * score (snapkv_score or rolekv_compress without lse_win) made on the calling
+ * thread so that the persistent score kernel's per-unit meeting point, where
+ * a unit's key chunks wait for each other between the two passes, waits for
+ * one arrival more than there are chunks -- one that never comes -- with a
+ * limit of limit_ns nanoseconds (1e3 .. 1e10) instead of the usual 2 s.  That
+ * call then gives up at the meeting point, ORs ROLEKV_STATUS_TIMEOUT into its
+ * status word, drains its copies and tensor-core work, frees its tensor
+ * memory and returns; its scores are not valid.  The arming is used up by
+ * that one call.  It lets a caller check, without a fault, that the real
+ * kernel's abort path reports the stuck wait and leaves the device usable. */
+int rolekv_selftest_score_timeout(int64_t limit_ns);
 
 #ifdef __cplusplus
 }

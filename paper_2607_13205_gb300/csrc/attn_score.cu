@@ -1170,8 +1170,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           __threadfence();
           atomicAdd(fa.work + 1 + u, 1);
           const uint64_t t0 = global_timer_ns();
-          while (ld_acquire_gpu(fa.work + 1 + u) < a.n_chunks) {
-            if (*sh.abort_flag || global_timer_ns() - t0 > kWaitLimitNs) {
+          while (ld_acquire_gpu(fa.work + 1 + u) < a.n_chunks + fa.hold) {
+            if (*sh.abort_flag || global_timer_ns() - t0 > fa.wait_ns) {
               *sh.abort_flag = 1;
               if (a.status) atomicOr(a.status, ROLEKV_STATUS_TIMEOUT);
               got = false;
@@ -1191,7 +1191,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int j = etid;
         const int p = row_position(a, n, rb, j);
         float nl = -INFINITY;
-        if (h2o) {
+        if (h2o && fa.single) {
+          // the caller's natural-log LSE of the query row (head g, position p)
+          if (p >= 0) {
+            const int g = j / a.P;
+            const int64_t hq = static_cast<int64_t>(un.h) * a.G + g;
+            const int64_t Hq = static_cast<int64_t>(a.Hkv) * a.G;
+            const int64_t o = a.varlen ? (un.l * Hq + hq) * a.T + un.tok0 + p
+                                       : ((static_cast<int64_t>(un.l) * a.b + un.s) * Hq + hq) * a.n_max + p;
+            nl = -__ldg(fa.h2o_lse + o) * kLog2e;
+          }
+        } else if (h2o) {
           const float2 ml = sh.merge[j];
           if (p >= 0 && ml.y > 0.f) nl = -(ml.x + log2f(ml.y));
         } else if (fa.single) {

@@ -6,13 +6,10 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include "internal.h"
 #include "rolekv.h"
 
 namespace rolekv {
-
-// Every device-side wait is bounded by this much wall time (globaltimer, ns);
-// when it runs out the kernel records ROLEKV_STATUS_TIMEOUT and unwinds.
-constexpr uint64_t kWaitLimitNs = 2000000000ull;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));

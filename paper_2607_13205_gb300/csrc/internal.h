@@ -12,6 +12,10 @@ namespace rolekv {
 
 enum { kModeSnapKV = 0, kModeH2O = 1 };
 
+// Every device-side wait is bounded by this much wall time (globaltimer, ns);
+// when it runs out the kernel records ROLEKV_STATUS_TIMEOUT and unwinds.
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+
 // Everything the two attention passes need, passed by value to the kernels.
 struct ScoreArgs {
   int32_t L, b, G, Hkv, d, n_max;
@@ -48,7 +52,13 @@ struct FusedArgs {
   ScoreArgs s;                      // s.n_chunks = chunks per unit, s.chunk_tiles = tiles per chunk
   int32_t* work;                    // [1 + u]: chunks of unit u done with pass 1 ([0] unused)
   int32_t n_items;
-  int32_t single;                   // 1: normalisers given in s.lse2, pass 2 only
+  int32_t single;                   // 1: pass 2 only; SnapKV normalisers given in s.lse2,
+                                    // H2O ones in h2o_lse
+  const float* h2o_lse;             // H2O, single: natural-log LSE of every query row
+                                    // (dense [L][b][Hq][n_max], varlen [L][Hq][T])
+  uint64_t wait_ns;                 // limit of the per-unit meeting point's wait
+  int32_t hold;                     // arrivals the meeting point waits for beyond the
+                                    // unit's chunks (0; 1 only in the timeout self-test)
 };
 
 cudaError_t launch_snapkv_fused(int d, const CUtensorMap& kmap, const CUtensorMap& qmap,

@@ -31,6 +31,12 @@ thread_local int g_stage_cursor = 0;
 
 void stage_begin() { g_stage_cursor = 0; }
 
+// Timeout self-test (rolekv_selftest_score_timeout): when armed, the next
+// two-pass SnapKV score on this thread waits at its per-unit meeting point for
+// one arrival more than there are chunks, with this limit.
+thread_local bool g_timeout_test_armed = false;
+thread_local uint64_t g_timeout_test_ns = 0;
+
 // Records the next stage event (if any) after a kernel launch.
 void stage_mark(cudaStream_t stream) {
   if (g_stage_cursor < g_num_stage_events) cudaEventRecord(g_stage_events[g_stage_cursor], stream);
@@ -305,11 +311,17 @@ int run_snapkv(const BatchInfo& bi, const int32_t* cu_seqlens, const rolekv_tens
   if (p.fused) {
     // one persistent launch: both passes with the normalisers formed
     // in-kernel, or pass 2 alone after the caller's normalisers are converted
-    FusedArgs fa;
+    FusedArgs fa{};
     fa.s = a;
     fa.work = p.work;
     fa.n_items = p.n_items;
     fa.single = lse_win != nullptr;
+    fa.wait_ns = kWaitLimitNs;
+    if (!fa.single && g_timeout_test_armed) {
+      fa.hold = 1;
+      fa.wait_ns = g_timeout_test_ns;
+      g_timeout_test_armed = false;
+    }
     if (fa.single) {
       e = launch_snapkv_lse(a, lse_win, stream);
       if (e != cudaSuccess) return cuda_fail(e, "snapkv normalisers");
@@ -564,8 +576,8 @@ int snapkv_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k
 }
 
 int h2o_score(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k, float scale,
-              float* scores, void* workspace, size_t workspace_bytes, int32_t* status_dev,
-              void* stream) {
+              const float* lse, float* scores, void* workspace, size_t workspace_bytes,
+              int32_t* status_dev, void* stream) {
   BatchInfo bi;
   int rc = check_batch(batch, &bi);
   if (rc) return rc;
@@ -574,6 +586,7 @@ int h2o_score(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k, float
   if (rc) return rc;
   if (bi.T == 0) return ROLEKV_OK;                 // no tokens: nothing to score
   if (scores == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "scores is NULL");
+  if (reinterpret_cast<uintptr_t>(lse) & 3u) return fail(ROLEKV_ERR_INVALID_ARG, "lse must be 4-byte aligned");
   if ((rc = check_tensor("q", q, bi.d, bi.Hq, bi.varlen, true))) return rc;
   if ((rc = check_tensor("k", k, bi.d, bi.Hkv, bi.varlen, true))) return rc;
   if ((rc = bind_workspace(p, workspace, workspace_bytes))) return rc;
@@ -595,13 +608,15 @@ int h2o_score(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k, float
   // every query block adds its column sums into the zeroed scores
   cudaError_t e = cudaMemsetAsync(scores, 0, static_cast<size_t>(score_elems(bi)) * sizeof(float), st);
   if (e != cudaSuccess) return cuda_fail(e, "clearing the scores");
-  // one persistent launch: per query block, its row normalisers (pass 1)
-  // then its share of the column sums (pass 2)
-  FusedArgs fa;
+  // one persistent launch: per query block, its row normalisers (pass 1, or
+  // the caller's LSE) then its share of the column sums (pass 2)
+  FusedArgs fa{};
   fa.s = a;
   fa.work = p.work;
   fa.n_items = p.n_items;
-  fa.single = 0;
+  fa.single = lse != nullptr;
+  fa.h2o_lse = lse;
+  fa.wait_ns = kWaitLimitNs;
   e = launch_snapkv_fused(bi.d, kmap, qmap, fa, st);
   if (e != cudaSuccess) return cuda_fail(e, "h2o fused score");
   stage_mark(st);
@@ -896,13 +911,14 @@ int snapkv_score_noalloc(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_
   if (rc) return rc;
   if (pool_k < 1 || pool_k > 15 || pool_k % 2 == 0)
     return fail(ROLEKV_ERR_UNSUPPORTED, "pool_k=%d must be odd, 1..15", pool_k);
+  ScorePlan p;
+  rc = plan_score(kModeSnapKV, bi, W, lse_win == nullptr, false, &p);
+  if (rc) return rc;
+  if (bi.T == 0) return ROLEKV_OK;                 // no tokens: nothing to score (as snapkv_score)
   if (scores == nullptr) return fail(ROLEKV_ERR_INVALID_ARG, "scores is NULL");
   if (pool_k > 1 && scores_prepool == nullptr)
     return fail(ROLEKV_ERR_INVALID_ARG,
                 "snapkv_score_noalloc with pool_k > 1 needs scores_prepool (the pre-pool output)");
-  ScorePlan p;
-  rc = plan_score(kModeSnapKV, bi, W, lse_win == nullptr, false, &p);
-  if (rc) return rc;
   if (p.bytes > kNoAllocScratchBytes)
     return fail(ROLEKV_ERR_UNSUPPORTED,
                 "batch needs %zu bytes of scratch; snapkv_score_noalloc holds at most %zu "
@@ -931,6 +947,14 @@ int snapkv_score_noalloc(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_
   cudaError_t e = launch_maxpool(p.a, pre, scores, pool_k, st);
   if (e != cudaSuccess) return cuda_fail(e, "max-pool");
   stage_mark(st);
+  return ROLEKV_OK;
+}
+
+int rolekv_selftest_score_timeout(int64_t limit_ns) {
+  if (limit_ns < 1000 || limit_ns > 10000000000LL)
+    return fail(ROLEKV_ERR_INVALID_ARG, "limit_ns=%lld outside 1e3..1e10", static_cast<long long>(limit_ns));
+  g_timeout_test_armed = true;
+  g_timeout_test_ns = static_cast<uint64_t>(limit_ns);
   return ROLEKV_OK;
 }
 

@@ -76,7 +76,8 @@ _SIGNATURES = [
       ctypes.c_void_p]),
     ("h2o_score", ctypes.c_int,
      [ctypes.POINTER(BatchDesc), Tensor, Tensor, ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p,
-      ctypes.c_size_t, ctypes.c_void_p, ctypes.c_void_p]),
+      ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p, ctypes.c_void_p]),
+    ("rolekv_selftest_score_timeout", ctypes.c_int, [ctypes.c_int64]),
     ("role_alloc_select", ctypes.c_int,
      [ctypes.POINTER(BatchDesc), ctypes.c_void_p, ctypes.c_void_p, ctypes.POINTER(SelectParams),
       ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
@@ -293,14 +294,22 @@ def decode_attention(batch: Batch, q: torch.Tensor, k_cache: torch.Tensor, v_cac
 
 
 def h2o_score(batch: Batch, q: torch.Tensor, k: torch.Tensor, scores: torch.Tensor, scale: float = 0.0,
-              ws: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None,
-              stream=None) -> torch.Tensor:
+              lse: Optional[torch.Tensor] = None, ws: Optional[torch.Tensor] = None,
+              status: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """lse: optional fp32 natural-log normalisers of every query row (dense
+    [L][b][Hq][n], varlen [L][Hq][T]); given, the score is one pass over K."""
     if ws is None:
         ws = workspace(OP_H2O, batch, 0, device=k.device)
     _check(lib().h2o_score(ctypes.byref(batch.desc), tensor_desc(q, batch.varlen),
-                           tensor_desc(k, batch.varlen), scale, _ptr(scores), _ptr(ws), ws.numel(),
-                           _ptr(status), _stream(stream)))
+                           tensor_desc(k, batch.varlen), scale, _ptr(lse), _ptr(scores), _ptr(ws),
+                           ws.numel(), _ptr(status), _stream(stream)))
     return scores
+
+
+def selftest_score_timeout(limit_ns: int) -> None:
+    """Arm the next two-pass SnapKV score on this thread to time out at its
+    per-unit meeting point after limit_ns (diagnostic; see rolekv.h)."""
+    _check(lib().rolekv_selftest_score_timeout(int(limit_ns)))
 
 
 def role_alloc_select(batch: Batch, scores: torch.Tensor, roles: torch.Tensor, params: SelectParams,

@@ -70,3 +70,54 @@ def check_index_sets(ob: O.Batch, u: int, got_idx: np.ndarray, ref_scores: np.nd
     for bk in range(n_roles):
         mem = buckets == bk
         assert sum(1 for t in g if mem[t]) == sum(1 for t in r if mem[t])
+
+
+def window_lse_oracle(w: I.Workload, ob: O.Batch, qb, kb) -> np.ndarray:
+    """Natural-log softmax normaliser of every SnapKV window row over its
+    causal keys, fp64 on the host from the bf16 inputs, stored as fp32
+    [L][b][Hq][W] (rows i >= W_eff left at 0): the LSE a prefill attention
+    hands over."""
+    lse = np.zeros((w.L, w.b, w.Hq, w.W), dtype=np.float32)
+    scale = 1.0 / np.sqrt(w.d)
+    for u in range(ob.n_units):
+        l, s, h = ob.unit(u)
+        k = O.bf16_to_f64(ob.kv_rows(kb, u))
+        n = k.shape[0]
+        if n == 0:
+            continue
+        w_eff = min(w.W, n)
+        for g in range(w.G):
+            q = O.bf16_to_f64(qb[l, s, h * w.G + g, :w_eff])
+            logits = scale * (q @ k.T)
+            for i in range(w_eff):
+                row = logits[i, :n - w_eff + i + 1]
+                m = row.max()
+                lse[l, s, h * w.G + g, i] = m + np.log(np.exp(row - m).sum())
+    return lse
+
+
+def prefill_lse_oracle(w: I.Workload, ob: O.Batch, qb, kb) -> np.ndarray:
+    """Natural-log softmax normaliser of every causal prefill query row, fp64
+    on the host from the bf16 inputs, stored as fp32 in the layout h2o_score
+    takes: dense [L][b][Hq][n_max], varlen [L][Hq][T]."""
+    shape = (w.L, w.Hq, ob.T) if w.varlen else (w.L, w.b, w.Hq, w.n)
+    lse = np.zeros(shape, dtype=np.float32)
+    scale = 1.0 / np.sqrt(w.d)
+    for u in range(ob.n_units):
+        l, s, h = ob.unit(u)
+        k = O.bf16_to_f64(ob.kv_rows(kb, u))
+        n = k.shape[0]
+        if n == 0:
+            continue
+        q = O.bf16_to_f64(ob.q_rows(qb, u))           # (G, n, d)
+        causal = np.arange(n)[None, :] <= np.arange(n)[:, None]
+        for g in range(w.G):
+            logits = np.where(causal, scale * (q[g] @ k.T), -np.inf)
+            m = logits.max(axis=1, keepdims=True)
+            row_lse = (m + np.log(np.exp(logits - m).sum(axis=1, keepdims=True)))[:, 0]
+            if w.varlen:
+                c0 = int(ob.cu[s])
+                lse[l, h * w.G + g, c0:c0 + n] = row_lse
+            else:
+                lse[l, s, h * w.G + g, :n] = row_lse
+    return lse

@@ -180,3 +180,45 @@ def test_struct_layouts_match_the_header(tmp_path):
         assert got[(st, "size")] == ctypes.sizeof(cls), st
         for f in fields[st]:
             assert got[(st, f)] == getattr(cls, f).offset, (st, f)
+
+
+_NOALLOC_REJECTS = r'''
+import ctypes, sys
+sys.path.insert(0, sys.argv[1])
+from paper_2607_13205_gb300 import rolekv as R
+lib = R.lib()
+t = R.Tensor(16, 0, 0, 0, 128)          # fake, never dereferenced: checks fail first
+f = ctypes.c_void_p(256)
+# 64 layers x 64 sequences x 8 KV heads at 16384 tokens need more scratch
+# than the static array holds
+b = R.BatchDesc(64, 64, 32, 8, 128, 16384, None, None)
+rc = lib.snapkv_score_noalloc(ctypes.byref(b), t, t, 32, 1, 0.0, None, f, None, None, None)
+assert rc == R.ERR_UNSUPPORTED, rc
+assert b"scratch" in lib.rolekv_last_error()
+# pooling without a pre-pool output buffer is refused too
+small = R.BatchDesc(1, 1, 8, 2, 128, 1000, None, None)
+rc = lib.snapkv_score_noalloc(ctypes.byref(small), t, t, 32, 7, 0.0, None, f, None, None, None)
+assert rc == R.ERR_INVALID_ARG, rc
+assert b"scores_prepool" in lib.rolekv_last_error()
+# so is a missing output; an empty batch needs none
+rc = lib.snapkv_score_noalloc(ctypes.byref(small), t, t, 32, 1, 0.0, None, None, None, None, None)
+assert rc == R.ERR_INVALID_ARG, rc
+empty = R.BatchDesc(1, 1, 8, 2, 128, 0, None, None)
+rc = lib.snapkv_score_noalloc(ctypes.byref(empty), t, t, 32, 7, 0.0, None, None, None, None, None)
+assert rc == R.OK, rc
+print("ok")
+'''
+
+
+def test_noalloc_rejects_on_the_host(lib):
+    """snapkv_score_noalloc refuses a batch larger than its static scratch and
+    pooling without a pre-pool buffer before any CUDA call.  Run in a child
+    process with every GPU hidden, so that even a validation regression could
+    only fail a CUDA call (a wrong return code), never touch a device."""
+    import subprocess
+    import sys
+    env = dict(os.environ, CUDA_VISIBLE_DEVICES="")
+    out = subprocess.run([sys.executable, "-c", _NOALLOC_REJECTS, B.ROOT], env=env,
+                         capture_output=True, text=True, timeout=300)
+    assert out.returncode == 0, out.stderr[-2000:]
+    assert out.stdout.strip().endswith("ok")

@@ -164,6 +164,31 @@ def test_long_context_full_size():
     _check_all_units(w, B, ob, r, 0.0, lambda n: min(w.W, n) * w.G)
     _check_sampled_snapkv(w, B, ob, [0, 517, ob.n_units - 1], r, 0.0)
     _check_ceil_select(w, B, r, [0, 517, ob.n_units - 1])
+    _check_one_call(w, B, ob, r, [5, 700, ob.n_units - 2])
+
+
+def _check_one_call(w, B, ob, r, units):
+    """rolekv_compress (score, select with the pool fused, compaction in one
+    call) on the same inputs: kept indices, per-role counts and compressed
+    K/V bit-exact against the three separate calls, and against the oracle on
+    the sampled units."""
+    batch = lib_batch(w, DEV)
+    params = R.select_params(B, I.PAPER_ALPHA, 0.0, I.ROLE_KEY)
+    keep = torch.full(batch.kept_shape(B), -7, dtype=torch.int32, device=DEV)
+    k_out = torch.empty(R.compact_shape(batch, B), dtype=torch.bfloat16, device=DEV)
+    v_out = torch.empty_like(k_out)
+    per_role = torch.empty((batch.n_units, I.N_ROLES), dtype=torch.int32, device=DEV)
+    ws = R.workspace(R.OP_COMPRESS, batch, w.W, device=DEV)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    R.rolekv_compress(batch, r["qw"], r["K"], r["V"], w.W, w.pool_k, torch.as_tensor(r["roles"], device=DEV),
+                      params, keep, k_out, v_out, ws, kept_per_role=per_role, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    assert np.array_equal(keep.cpu().numpy(), r["keep"])
+    assert np.array_equal(per_role.cpu().numpy(), r["per_role"])
+    assert torch.equal(k_out, r["k_out"]) and torch.equal(v_out, r["v_out"])
+    r1 = dict(r, keep=keep.cpu().numpy(), k_out=k_out, v_out=v_out)
+    _check_sampled_snapkv(w, B, ob, units, r1, 0.0)
 
 
 @pytest.mark.parametrize("B", I.WORKLOADS["llama8b"].budgets)

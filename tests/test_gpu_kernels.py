@@ -9,7 +9,8 @@ import torch
 from oracle import rolekv_oracle as O
 from paper_2607_13205_gb300 import inputs as I
 from paper_2607_13205_gb300 import rolekv as R
-from tests.gpu_helpers import assert_scores_close, check_index_sets, lib_batch, oracle_batch
+from tests.gpu_helpers import (assert_scores_close, check_index_sets, lib_batch, oracle_batch,
+                               prefill_lse_oracle, window_lse_oracle)
 
 pytestmark = pytest.mark.gpu
 
@@ -59,6 +60,24 @@ def test_snapkv_score_matches_oracle(case):
             assert abs(ob.score_view(gpre, u).astype(np.float64).sum() - min(w.W, n) * w.G) < 1e-3 * min(w.W, n) * w.G
 
 
+@pytest.mark.parametrize("pool_k", [5, 11])
+@pytest.mark.parametrize("case", ["ragged_tail_g4w32", "varlen_short_empty"])
+def test_snapkv_score_pool_widths(case, pool_k):
+    """The standalone max-pool at the paper's other swept widths (Section 4),
+    dense and varlen (pools never cross a sequence boundary)."""
+    w = SNAPKV_CASES[case]
+    roles, K, V, qw = _snapkv_inputs(w, seed=5)
+    batch = lib_batch(w, DEV)
+    scores = torch.full(batch.score_shape(), -1.0, dtype=torch.float32, device=DEV)
+    R.snapkv_score(batch, qw, K, w.W, pool_k, scores)
+    torch.cuda.synchronize()
+    ob = oracle_batch(w)
+    ref = O.snapkv_batch(ob, I.bf16_bits(qw), I.bf16_bits(K), w.W, pool_k)
+    got = scores.cpu().numpy()
+    for u, (_, rpool) in ref.items():
+        assert_scores_close(ob.score_view(got, u), rpool, f"{case} pool {pool_k} unit {u}")
+
+
 @pytest.mark.parametrize("scale", [0.004, 0.5])
 @pytest.mark.parametrize("case", ["two_row_tiles_w64_multichunk", "varlen_g7"])
 def test_snapkv_and_h2o_with_explicit_scale(case, scale):
@@ -91,29 +110,15 @@ def test_snapkv_and_h2o_with_explicit_scale(case, scale):
         assert_scores_close(obh.score_view(hgot, u), r, f"{case} scale {scale} unit {u} h2o")
 
 
-@pytest.mark.parametrize("case", ["varlen_short_empty", "two_row_tiles_w64_multichunk"])
+@pytest.mark.parametrize("case", ["varlen_short_empty", "two_row_tiles_w64_multichunk", "varlen_g7"])
 def test_snapkv_with_supplied_lse(case):
-    """Single pass with the window rows' normalisers given (natural log)."""
+    """Single pass with the window rows' normalisers given (natural log, fp32,
+    from the oracle's fp64 logits)."""
     w = SNAPKV_CASES[case]
     roles, K, V, qw = _snapkv_inputs(w, seed=3)
     ob = oracle_batch(w)
     kb, qb = I.bf16_bits(K), I.bf16_bits(qw)
-    lse = np.zeros((w.L, w.b, w.Hq, w.W), dtype=np.float32)
-    scale = 1.0 / np.sqrt(w.d)
-    for u in range(ob.n_units):
-        l, s, h = ob.unit(u)
-        k = O.bf16_to_f64(ob.kv_rows(kb, u))
-        n = k.shape[0]
-        if n == 0:
-            continue
-        w_eff = min(w.W, n)
-        for g in range(w.G):
-            q = O.bf16_to_f64(qb[l, s, h * w.G + g, :w_eff])
-            logits = scale * (q @ k.T)
-            for i in range(w_eff):
-                row = logits[i, :n - w_eff + i + 1]
-                m = row.max()
-                lse[l, s, h * w.G + g, i] = m + np.log(np.exp(row - m).sum())
+    lse = window_lse_oracle(w, ob, qb, kb)
     batch = lib_batch(w, DEV)
     scores = torch.empty(batch.score_shape(), dtype=torch.float32, device=DEV)
     R.snapkv_score(batch, qw, K, w.W, w.pool_k, scores, lse_win=torch.as_tensor(lse, device=DEV))
@@ -121,9 +126,7 @@ def test_snapkv_with_supplied_lse(case):
     ref = O.snapkv_batch(ob, qb, kb, w.W, w.pool_k)
     got = scores.cpu().numpy()
     for u, (_, rpool) in ref.items():
-        # the normaliser is rounded to fp32 once more here: 2e-3 covers it
-        g = ob.score_view(got, u).astype(np.float64)
-        assert np.all(np.abs(g - rpool) <= 2e-3 * np.abs(rpool) + 1e-20), f"unit {u}"
+        assert_scores_close(ob.score_view(got, u), rpool, f"{case} unit {u}")
 
 
 H2O_CASES = {
@@ -151,6 +154,34 @@ def test_h2o_score_matches_oracle(case):
         assert_scores_close(ob.score_view(got, u), s, f"{case} unit {u}")
         if s.size:
             assert abs(ob.score_view(got, u).astype(np.float64).sum() - s.size * w.G) < 1e-3 * s.size * w.G
+
+
+@pytest.mark.parametrize("case", list(H2O_CASES))
+def test_h2o_score_with_supplied_lse(case):
+    """One pass over K with every query row's natural-log normaliser given
+    (fp32, from the oracle's fp64 logits; dense [L][b][Hq][n], varlen
+    [L][Hq][T]): against the oracle, and against the two-pass score."""
+    w = H2O_CASES[case]
+    roles = I.workload_roles(w, 2)
+    K, _ = I.make_kv(w, roles, 2, device=DEV, with_v=False)
+    Q = I.make_q_full(w, 2, device=DEV)
+    batch = lib_batch(w, DEV)
+    ob = oracle_batch(w)
+    qb, kb = I.bf16_bits(Q), I.bf16_bits(K)
+    lse = torch.as_tensor(prefill_lse_oracle(w, ob, qb, kb), device=DEV)
+    one = torch.full(batch.score_shape(), -1.0, dtype=torch.float32, device=DEV)
+    two = torch.full_like(one, -1.0)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    R.h2o_score(batch, Q, K, one, lse=lse, status=status)
+    R.h2o_score(batch, Q, K, two, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    ref = O.h2o_batch(ob, qb, kb)
+    g1, g2 = one.cpu().numpy(), two.cpu().numpy()
+    for u, s in ref.items():
+        assert_scores_close(ob.score_view(g1, u), s, f"{case} unit {u} one pass")
+        assert_scores_close(ob.score_view(g1, u), ob.score_view(g2, u).astype(np.float64),
+                            f"{case} unit {u} one pass against two")
 
 
 # -------------------------------------------------------------------- quest
@@ -340,6 +371,9 @@ SELECT_CASES = [
     ("varlen", VARLEN4, 0.10, 0.0, 0, 0, 7),
     ("mid_n", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=12001), 0.10, 0.02, 0, 0, 7),
     ("mid_n_global_pool15", _w("llama8b", L=1, b=1, Hq=4, Hkv=1, n=9999), 0.10, 0.0, 1, 0, 15),
+    # the paper's other swept pool widths (Section 4: 3, 5, 7, 11, 15)
+    ("combined_pool11", _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=5000), 0.10, 0.02, 0, 0, 11),
+    ("varlen_global_pool11", VARLEN4, 0.20, 0.0, 1, 0, 11),
     ("max_n", _w("long", L=1, b=1, Hq=4, Hkv=1, n=R.SELECT_MAX_N), 0.10, 0.0, 0, 0, 7),
     # fair eviction (equal retention rate per role) and the recency floor
     ("fair_pool7", _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=5000), 0.10, 0.0, R.POLICY_FAIR, 0, 7),
@@ -688,6 +722,39 @@ def test_bounded_wait_reports_timeout():
     assert 0.015 <= dt < 5.0
     x = torch.arange(8, device=DEV).sum()        # the context still works
     assert int(x.item()) == 28
+
+
+@pytest.mark.parametrize("case", ["two_row_tiles_w64_multichunk", "varlen_short_empty"])
+def test_fused_score_meeting_point_timeout(case):
+    """The persistent score kernel's own abort path: armed by the self-test,
+    its per-unit meeting point waits for an arrival that never comes, gives up
+    after 30 ms, reports STATUS_TIMEOUT and returns (its copies drained, its
+    tensor memory freed).  The next call on the same device and stream runs
+    normally and matches the oracle."""
+    import time
+    w = SNAPKV_CASES[case]
+    roles, K, V, qw = _snapkv_inputs(w, seed=12)
+    batch = lib_batch(w, DEV)
+    scores = torch.full(batch.score_shape(), -1.0, dtype=torch.float32, device=DEV)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    R.selftest_score_timeout(30_000_000)
+    R.snapkv_score(batch, qw, K, w.W, 1, scores, status=status)
+    torch.cuda.synchronize()
+    dt = time.perf_counter() - t0
+    assert int(status.item()) & R.STATUS_TIMEOUT
+    assert 0.025 <= dt < 10.0
+    # the arming is used up: the next call is a normal one
+    status.zero_()
+    R.snapkv_score(batch, qw, K, w.W, 1, scores, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    ob = oracle_batch(w)
+    ref = O.snapkv_batch(ob, I.bf16_bits(qw), I.bf16_bits(K), w.W, 1)
+    got = scores.cpu().numpy()
+    for u, (rpre, _) in ref.items():
+        assert_scores_close(ob.score_view(got, u), rpre, f"{case} unit {u} after the timeout")
 
 
 @pytest.mark.parametrize("varlen", [False, True])

@@ -88,7 +88,7 @@ extern "C" {
 #define ROLEKV_POLICY_CEIL 4        /* Algorithm 1's ceilings taken literally  */
 
 #define ROLEKV_MAX_ROLES 8
-#define ROLEKV_SELECT_MAX_N 40960   /* largest sequence role_alloc_select takes */
+#define ROLEKV_SELECT_MAX_N 262144  /* largest sequence role_alloc_select takes */
 
 typedef struct rolekv_tensor {
   const void* ptr;
@@ -297,7 +297,10 @@ int h2o_score(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k, float
  *   keep_idx      int32 kept-index array (ascending positions, -1 padded).
  *   keep_mask     optional uint8 array in the score layout: 1 kept, 0 evicted.
  *   kept_per_role optional int32 [units][n_roles]: kept tokens per role.
- * Sequences longer than ROLEKV_SELECT_MAX_N are rejected (ERR_UNSUPPORTED). */
+ * Sequences longer than ROLEKV_SELECT_MAX_N are rejected (ERR_UNSUPPORTED).
+ * Rows of up to 40960 tokens keep their pooled keys in shared memory; longer
+ * rows recompute them from the score row on each pass (the same kept set,
+ * more reads of the scores from L2). */
 int role_alloc_select(const rolekv_batch* batch, const float* scores, const uint8_t* roles,
                       const rolekv_select_params* params, int32_t pool_k, int32_t* keep_idx,
                       uint8_t* keep_mask, int32_t* kept_per_role, int32_t* status_dev,

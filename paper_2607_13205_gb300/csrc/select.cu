@@ -29,6 +29,10 @@
 // A unit with a NaN, keys of both signs, or more candidates than the list
 // holds 4 to 5 bits above the bottom takes the general path: four 8-bit
 // rounds over all slots.
+// Rows longer than kSmemMaxN tokens (streaming mode) do not keep their keys:
+// every pass recomputes a group's pooled keys from the score row (read again
+// from L2), the first-digit histograms count in 32 bits and a candidate-list
+// entry carries its key beside (bucket << 24) | slot.
 // Kept positions are then written in ascending order from a block-wide scan
 // of the bit words.
 #include <cuda_runtime.h>
@@ -48,6 +52,10 @@ constexpr uint32_t kCodeDrop = 0x80;   // no bucket keeps the token
 // codes 0 .. kR-1: the token's bucket keeps only keys above a threshold
 constexpr int kTieCap = 256;           // ranked ties held in shared memory
 
+// Longest row whose keys a CTA holds in shared memory; longer rows take the
+// streaming mode.
+constexpr int kSmemMaxN = 40960;
+
 // Groups (of four slots) reserved per CTA: n_max tokens plus up to three
 // leading slots, rounded to a multiple of 32 groups so that the bit words
 // (one per 8 groups) end on a 16-byte boundary.
@@ -55,9 +63,10 @@ __host__ __device__ inline int select_groups(int n_max) { return (((n_max + 3 + 
 // Width of the first digit: 2^NB bins per role.
 __host__ __device__ inline int first_digit_bits(int n_max) { return n_max > 16384 ? 11 : 10; }
 // Bytes of the region that holds the pass-1 histograms (8 roles x 2^NB bins
-// x 16-bit counts), reused for the candidate list (4-byte entries).
+// x 16-bit counts; 32-bit in streaming mode, where a bin can pass 65535),
+// reused for the candidate list (4-byte entries; 8-byte in streaming mode).
 __host__ __device__ inline size_t region_bytes(int n_max) {
-  return static_cast<size_t>(kR) * (size_t{1} << first_digit_bits(n_max)) * 2;
+  return static_cast<size_t>(kR) * (size_t{1} << first_digit_bits(n_max)) * (n_max > kSmemMaxN ? 4 : 2);
 }
 
 // Monotone map of a float to uint32 (larger float -> larger key); -0 is folded
@@ -161,7 +170,7 @@ __device__ __forceinline__ uint32_t floor_bits(int s0, int nf, int n) {
 }
 
 // Pass 1 for a pool half-width HW known at compile time.
-template <int HW, int NT, bool GL>
+template <int HW, int NT, bool GL, bool STREAM>
 __device__ __forceinline__ void pass1(const UnitView& v, int n_roles, uint32_t ban, int nb,
                                       uint4* keys4, uint32_t* hist16, int32_t* floor_role,
                                       bool& nan_hint, uint32_t& top_and, uint32_t& top_or) {
@@ -197,7 +206,7 @@ __device__ __forceinline__ void pass1(const UnitView& v, int n_roles, uint32_t b
       }
       k[j] = ordered_key(m);
     }
-    keys4[g] = make_uint4(k[0], k[1], k[2], k[3]);
+    if (!STREAM) keys4[g] = make_uint4(k[0], k[1], k[2], k[3]);
     const uint32_t fb = floor_bits(4 * g - v.off, v.nf, v.n);
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
@@ -208,11 +217,46 @@ __device__ __forceinline__ void pass1(const UnitView& v, int n_roles, uint32_t b
         top_and &= k[j];
         top_or |= k[j];
         const uint32_t bin = (k[j] >> sh0) & bmask;
-        if (!GL || !((ban >> r) & 1u))
-          atomicAdd(&hist16[(GL ? 0u : r) * words_per_role + (bin >> 1)], 1u << (16 * (bin & 1u)));
+        if (!GL || !((ban >> r) & 1u)) {
+          if (STREAM)
+            atomicAdd(&hist16[((GL ? 0u : r) << nb) + bin], 1u);   // 32-bit bins
+          else
+            atomicAdd(&hist16[(GL ? 0u : r) * words_per_role + (bin >> 1)], 1u << (16 * (bin & 1u)));
+        }
       }
     }
   }
+}
+
+// Streaming mode: the four keys of group g recomputed from the score row, the
+// same max-pool as pass 1 (stride 1, -inf outside the row, half-width hw);
+// nan_aware: a window holding a NaN gives key 0 (below every other key).
+__device__ __forceinline__ uint4 stream_group_keys(const UnitView& v, int g, int hw, bool nan_aware) {
+  float x[20];
+#pragma unroll
+  for (int o = -2; o <= 2; ++o) {
+    const float4 f = load_slots(v.sp, v.off, v.n, g + o);
+    x[4 * (o + 2) + 0] = f.x;
+    x[4 * (o + 2) + 1] = f.y;
+    x[4 * (o + 2) + 2] = f.z;
+    x[4 * (o + 2) + 3] = f.w;
+  }
+  uint32_t k[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    float m = x[8 + j];
+    bool nanw = m != m;
+#pragma unroll
+    for (int d = 1; d <= 7; ++d) {
+      if (d <= hw) {
+        const float lo = x[8 + j - d], hi = x[8 + j + d];
+        nanw |= (lo != lo) | (hi != hi);
+        m = max3f(m, lo, hi);
+      }
+    }
+    k[j] = (nan_aware && nanw) ? 0u : ordered_key(m);
+  }
+  return make_uint4(k[0], k[1], k[2], k[3]);
 }
 
 // Quotas of one sequence by warp 0, lane r for role r: water-filling of the
@@ -436,6 +480,69 @@ __device__ void descend_first(const SelectArgs& a, SelShared& S, const uint32_t*
   }
 }
 
+// descend_first for the streaming mode's 32-bit bins: lane L owns bins
+// L * 2^NB / 32 ..; the lanes' totals locate the lane holding the threshold,
+// then the warp splits that lane's bins (at most 64, two per lane).
+template <int NB>
+__device__ void descend_first32(const SelectArgs& a, SelShared& S, const uint32_t* hist32, int b,
+                                int lane) {
+  constexpr int bpl = 1 << (NB - 5);   // bins per lane
+  const uint32_t* h0 = hist32 + (b << NB);
+  int mine = 0;
+#pragma unroll 8
+  for (int i = 0; i < bpl; ++i) mine += static_cast<int>(h0[lane * bpl + ((i + lane) & (bpl - 1))]);
+  int incl = mine;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int v = __shfl_down_sync(0xffffffffu, incl, o);
+    if (lane + o < 32) incl += v;
+  }
+  const int above = incl - mine;
+  const int need = S.need[b];
+  const unsigned who = __ballot_sync(0xffffffffu, above < need && above + mine >= need);
+  if (who == 0) {
+    if (lane == 0) S.general = 1;
+    return;
+  }
+  const int F = __ffs(who) - 1;
+  const int aboveF = __shfl_sync(0xffffffffu, above, F);
+  const int needF = need - aboveF;
+  // lane L takes bins F * bpl + 2L, 2L + 1 (descending order: the higher bin first)
+  const int i0 = 2 * lane;
+  const int lo = i0 < bpl ? static_cast<int>(h0[F * bpl + i0]) : 0;
+  const int hi = i0 + 1 < bpl ? static_cast<int>(h0[F * bpl + i0 + 1]) : 0;
+  const int pair = lo + hi;
+  int incl2 = pair;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int v = __shfl_down_sync(0xffffffffu, incl2, o);
+    if (lane + o < 32) incl2 += v;
+  }
+  const int above2 = incl2 - pair;
+  const unsigned who2 = __ballot_sync(0xffffffffu, above2 < needF && above2 + pair >= needF);
+  if (who2 == 0) {
+    if (lane == 0) S.general = 1;
+    return;
+  }
+  if (lane == __ffs(who2) - 1) {
+    const int bin0 = F * bpl + i0;
+    int fd, gb, ad;
+    if (above2 + hi >= needF) {
+      fd = bin0 + 1;
+      gb = aboveF + above2;
+      ad = hi;
+    } else {
+      fd = bin0;
+      gb = aboveF + above2 + hi;
+      ad = lo;
+    }
+    const int sh0 = 31 - NB;
+    S.prefix[b] = (S.top_and & 0x80000000u) | (static_cast<uint32_t>(fd) << sh0);
+    S.need[b] = need - gb;
+    S.cand[b] = ad;
+  }
+}
+
 // Exclusive prefix, in slot order, of popc(mask_of(q)) over the bit words
 // q < nwords: warp w walks a contiguous range of words (a multiple of 32), the
 // warps' totals are combined through shared memory, and body(q, mask, rank of
@@ -485,7 +592,7 @@ __device__ __forceinline__ void store_bits(uint32_t* bits, int g, int nwords, in
   if ((lane & 7) == 0 && g < 8 * nwords) bits[g >> 3] = x;
 }
 
-template <int NT>
+template <int NT, bool STREAM>
 __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs a) {
   constexpr int NW = NT / 32;
   extern __shared__ __align__(16) uint8_t dyn[];
@@ -527,14 +634,22 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
   const int iters = (ngroups + NT - 1) / NT;
   const int nb = first_digit_bits(a.n_max);
   const int groups_alloc = select_groups(a.n_max);
+  // keys (in-memory mode only), keep bits, then the histogram / list region
   uint4* keys4 = reinterpret_cast<uint4*>(dyn);
   const uint32_t* keys = reinterpret_cast<const uint32_t*>(keys4);
-  uint32_t* bits = reinterpret_cast<uint32_t*>(dyn + static_cast<size_t>(groups_alloc) * 16);
+  uint32_t* bits = reinterpret_cast<uint32_t*>(dyn + (STREAM ? 0 : static_cast<size_t>(groups_alloc) * 16));
   uint32_t* region = bits + groups_alloc / 8;   // 16-byte aligned (groups_alloc % 32 == 0)
   uint32_t* hist16 = region;                    // pass 1 histograms
   uint32_t* list = region;                      // then the candidate list
-  const int list_cap = static_cast<int>(region_bytes(a.n_max) / 4);
+  const int list_cap = static_cast<int>(region_bytes(a.n_max) / (STREAM ? 8 : 4));
   const bool global = a.policy == ROLEKV_POLICY_GLOBAL;
+  const int hw = a.pool_k / 2;
+  // a group's four keys: held (in-memory mode) or recomputed from the scores
+  bool nan_keys = false;                        // streaming mode: NaN windows give key 0
+  auto kv_of = [&](int g) -> uint4 {
+    if constexpr (STREAM) return stream_group_keys(v, g, hw, nan_keys);
+    else return keys4[g];
+  };
 
   if (tid < kR) {
     S.count[tid] = 0;
@@ -583,11 +698,11 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
     uint32_t tand = 0xFFFFFFFFu, tor = 0u;
     // GLOBAL: one histogram (row 0) of every eligible token; otherwise one
     // row per role
-#define ROLEKV_PASS1(HWV)                                                                   \
-  (global ? pass1<HWV, NT, true>(v, a.n_roles, a.ban_mask, nb, keys4, hist16, S.floor_role, \
-                                 nan_hint, tand, tor)                                       \
-          : pass1<HWV, NT, false>(v, a.n_roles, a.ban_mask, nb, keys4, hist16, S.floor_role, \
-                                  nan_hint, tand, tor))
+#define ROLEKV_PASS1(HWV)                                                                           \
+  (global ? pass1<HWV, NT, true, STREAM>(v, a.n_roles, a.ban_mask, nb, keys4, hist16, S.floor_role, \
+                                         nan_hint, tand, tor)                                       \
+          : pass1<HWV, NT, false, STREAM>(v, a.n_roles, a.ban_mask, nb, keys4, hist16, S.floor_role, \
+                                          nan_hint, tand, tor))
     switch (a.pool_k >> 1) {
       case 0: ROLEKV_PASS1(0); break;
       case 1: ROLEKV_PASS1(1); break;
@@ -613,17 +728,25 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
   // Role counts: the sums of the roles' histograms (a warp's 32 words belong
   // to one role); GLOBAL: the eligible total, in count[0].
   {
-    const int wpr = 1 << (nb - 1);
+    const int wpr = STREAM ? (1 << nb) : (1 << (nb - 1));   // words per role
+    const int lwpr = STREAM ? nb : nb - 1;
     for (int x0 = warp * 32; x0 < (global ? 1 : a.n_roles) * wpr; x0 += NT) {
       const uint32_t w = hist16[x0 + lane];
-      const int c = warp_sum(static_cast<int>((w & 0xFFFFu) + (w >> 16)));
-      if (lane == 0 && c) atomicAdd(&S.count[x0 >> (nb - 1)], c);
+      const int c = warp_sum(STREAM ? static_cast<int>(w) : static_cast<int>((w & 0xFFFFu) + (w >> 16)));
+      if (lane == 0 && c) atomicAdd(&S.count[x0 >> lwpr], c);
     }
   }
 
   // A NaN score (or +inf and -inf in one group): redo the keys one token at a
-  // time, a window holding a NaN giving the lowest key.
-  if (S.nan_hint) {
+  // time, a window holding a NaN giving the lowest key (streaming mode: every
+  // later recomputation of the keys does so).
+  if (STREAM) nan_keys = S.nan_hint != 0;
+  if (STREAM && S.nan_hint) {
+    bool seen = false;
+    for (int t = tid; t < n; t += NT) seen |= isnan(__ldg(v.sp + t));
+    if (__any_sync(0xffffffffu, seen) && lane == 0) S.nan_seen = 1;
+  }
+  if (!STREAM && S.nan_hint) {
     const int hw = a.pool_k / 2;
     uint32_t* kw = reinterpret_cast<uint32_t*>(keys4);
     bool seen = false;
@@ -661,7 +784,9 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
   // ---- first digit per bucket
   if (any_thr && !S.general) {
     if (warp < kR && S.mode[warp] == 2) {
-      if (nb == 11)
+      if (STREAM)
+        descend_first32<11>(a, S, hist16, warp, lane);
+      else if (nb == 11)
         descend_first<11>(a, S, hist16, warp, lane);
       else
         descend_first<10>(a, S, hist16, warp, lane);
@@ -682,7 +807,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
       for (int i = 0; i < iters; ++i) {
         const int g = i * NT + tid;
         if (g >= ngroups) break;
-        const uint4 kv = keys4[g];
+        const uint4 kv = kv_of(g);
         const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
         const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
         const uint32_t fb = floor_bits(4 * g - off, v.nf, n);
@@ -726,9 +851,13 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
       r_after = roles_of(i + 2);
       uint32_t m4 = 0, c4 = 0;
       uint32_t ent[4] = {0u, 0u, 0u, 0u};
+      uint32_t kk[4] = {0u, 0u, 0u, 0u};
       if (g < ngroups) {
-        const uint4 kv = keys4[g];
-        const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
+        const uint4 kv = kv_of(g);
+        kk[0] = kv.x;
+        kk[1] = kv.y;
+        kk[2] = kv.z;
+        kk[3] = kv.w;
         const uint32_t fb = floor_bits(4 * g - off, v.nf, n);
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
@@ -738,7 +867,8 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
           m4 |= static_cast<uint32_t>(hb > T) << j;
           if (hb == T && !((fb >> j) & 1u)) {
             c4 |= 1u << j;
-            ent[j] = (static_cast<uint32_t>(S.code_of_role[r]) << 16) | static_cast<uint32_t>(4 * g + j);
+            ent[j] = (static_cast<uint32_t>(S.code_of_role[r]) << (STREAM ? 24 : 16)) |
+                     static_cast<uint32_t>(4 * g + j);
           }
         }
         m4 |= fb;                                  // the recency floor is kept
@@ -759,7 +889,14 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
 #pragma unroll
         for (int j = 0; j < 4; ++j)
           if ((c4 >> j) & 1u) {
-            if (pos < list_cap) list[pos] = ent[j];
+            if (pos < list_cap) {
+              if (STREAM) {
+                list[2 * pos] = kk[j];
+                list[2 * pos + 1] = ent[j];
+              } else {
+                list[pos] = ent[j];
+              }
+            }
             ++pos;
           }
       }
@@ -779,9 +916,9 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
         const int d = lo < 8 ? lo : 8;
         const int shift = lo - d;
         for (int e = tid; e < m; e += NT) {
-          const uint32_t ent = list[e];
-          const uint32_t c = ent >> 16;
-          const uint32_t key = keys[ent & 0xFFFFu];
+          const uint32_t ent = STREAM ? list[2 * e + 1] : list[e];
+          const uint32_t c = STREAM ? ent >> 24 : ent >> 16;
+          const uint32_t key = STREAM ? list[2 * e] : keys[ent & 0xFFFFu];
           if ((key >> lo) == (S.prefix[c] >> lo))
             atomicAdd(&S.hist[c][(key >> shift) & ((1u << d) - 1u)], 1);
         }
@@ -793,9 +930,10 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
       // kept candidates join the bits; ties of partial buckets are gathered
       const uint32_t partial = S.partial_ties;
       for (int e = tid; e < m; e += NT) {
-        const uint32_t ent = list[e];
-        const uint32_t c = ent >> 16, slot = ent & 0xFFFFu;
-        const uint32_t key = keys[slot];
+        const uint32_t ent = STREAM ? list[2 * e + 1] : list[e];
+        const uint32_t c = STREAM ? ent >> 24 : ent >> 16;
+        const uint32_t slot = STREAM ? ent & 0xFFFFFFu : ent & 0xFFFFu;
+        const uint32_t key = STREAM ? list[2 * e] : keys[slot];
         if (key >= S.thr[c]) {
           atomicOr(&bits[slot >> 5], 1u << (slot & 31u));
         } else if (((partial >> c) & 1u) && key == S.prefix[c]) {
@@ -807,13 +945,15 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
       const int nt = S.tie_n;
       if (partial != 0 && nt <= kTieCap) {
         // index-order rank among the bucket's ties
+        constexpr int kCodeShift = STREAM ? 24 : 16;
+        constexpr uint32_t kSlotMask = STREAM ? 0xFFFFFFu : 0xFFFFu;
         for (int t = tid; t < nt; t += NT) {
           const uint32_t ent = S.ties[t];
-          const uint32_t c = ent >> 16, slot = ent & 0xFFFFu;
+          const uint32_t c = ent >> kCodeShift, slot = ent & kSlotMask;
           int rank = 0;
           for (int x = 0; x < nt; ++x) {
             const uint32_t o = S.ties[x];
-            rank += ((o >> 16) == c && (o & 0xFFFFu) < slot);
+            rank += ((o >> kCodeShift) == c && (o & kSlotMask) < slot);
           }
           if (rank < S.need[c]) atomicOr(&bits[slot >> 5], 1u << (slot & 31u));
         }
@@ -836,7 +976,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
       for (int i = 0; i < iters; ++i) {
         const int g = i * NT + tid;
         if (g >= ngroups) break;
-        const uint4 kv = keys4[g];
+        const uint4 kv = kv_of(g);
         const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
         const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
         const uint32_t fb = floor_bits(4 * g - off, v.nf, n);
@@ -856,7 +996,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
       const int g = i * NT + tid;
       uint32_t m4 = 0;
       if (g < ngroups) {
-        const uint4 kv = keys4[g];
+        const uint4 kv = kv_of(g);
         const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
         const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
 #pragma unroll
@@ -885,7 +1025,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
         for (int gg = 0; gg < 8; ++gg) {
           const int g = 8 * q + gg;
           if (g >= ngroups) break;
-          const uint4 kv = keys4[g];
+          const uint4 kv = kv_of(g);
           const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
           const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
           const uint32_t fb = floor_bits(4 * g - off, v.nf, n);
@@ -933,7 +1073,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
       for (int i = 0; i < iters; ++i) {
         const int g = i * NT + tid;
         if (g >= ngroups) break;
-        const uint4 kv = keys4[g];
+        const uint4 kv = kv_of(g);
         const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
         const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
         const uint32_t fb = floor_bits(4 * g - off, v.nf, n);
@@ -956,7 +1096,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
     for (int i = 0; i < iters; ++i) {
       const int g = i * NT + tid;
       if (g >= ngroups) break;
-      const uint4 kv = keys4[g];
+      const uint4 kv = kv_of(g);
       const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
       const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
       const uint32_t fb = floor_bits(4 * g - off, v.nf, n);
@@ -974,7 +1114,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
         for (int gg = 0; gg < 8; ++gg) {
           const int g = 8 * q + gg;
           if (g >= ngroups) break;
-          const uint4 kv = keys4[g];
+          const uint4 kv = kv_of(g);
           const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
           const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
           const uint32_t fb = floor_bits(4 * g - off, v.nf, n);
@@ -1045,12 +1185,12 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
   if (tid == 0 && S.nan_seen && a.status != nullptr) atomicOr(a.status, ROLEKV_STATUS_NONFINITE);
 }
 
-template <int NT>
+template <int NT, bool STREAM>
 cudaError_t launch_select_nt(const SelectArgs& a, size_t smem, cudaStream_t stream) {
-  cudaError_t e = cudaFuncSetAttribute(select_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(select_kernel<NT, STREAM>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  select_kernel<NT><<<a.n_units, NT, smem, stream>>>(a);
+  select_kernel<NT, STREAM><<<a.n_units, NT, smem, stream>>>(a);
   return cudaGetLastError();
 }
 
@@ -1058,7 +1198,7 @@ cudaError_t launch_select_nt(const SelectArgs& a, size_t smem, cudaStream_t stre
 
 size_t select_smem_bytes(int n_max) {
   const size_t groups = static_cast<size_t>(select_groups(n_max));
-  return groups * 16 + groups / 8 * 4 + region_bytes(n_max);
+  return (n_max > kSmemMaxN ? 0 : groups * 16) + groups / 8 * 4 + region_bytes(n_max);
 }
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream) {
@@ -1066,9 +1206,10 @@ cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream) {
   const size_t smem = select_smem_bytes(a.n_max);
   // CTA size follows the row length so that short rows still fill the SM
   // with several CTAs (shared memory is sized by the longest row).
-  if (a.n_max > 16384) return launch_select_nt<1024>(a, smem, stream);
-  if (a.n_max > 8192) return launch_select_nt<512>(a, smem, stream);
-  return launch_select_nt<256>(a, smem, stream);
+  if (a.n_max > kSmemMaxN) return launch_select_nt<1024, true>(a, smem, stream);
+  if (a.n_max > 16384) return launch_select_nt<1024, false>(a, smem, stream);
+  if (a.n_max > 8192) return launch_select_nt<512, false>(a, smem, stream);
+  return launch_select_nt<256, false>(a, smem, stream);
 }
 
 }  // namespace rolekv

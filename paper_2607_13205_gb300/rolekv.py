@@ -20,7 +20,7 @@ OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA = 0, 1, 2, 3, 4
 STATUS_NONFINITE, STATUS_BAD_INDEX, STATUS_TIMEOUT = 1, 2, 4
 POLICY_ROLE_QUOTA, POLICY_GLOBAL, POLICY_FAIR, POLICY_SLACK, POLICY_CEIL = 0, 1, 2, 3, 4
 MAX_ROLES = 8
-SELECT_MAX_N = 40960
+SELECT_MAX_N = 262144
 OP_SNAPKV, OP_H2O, OP_COMPRESS = 0, 1, 2
 
 

@@ -359,6 +359,10 @@ def _tied_scores(shape, seed):
 
 
 VARLEN4 = _w("ragged", L=2, b=4, Hq=8, Hkv=2, n=3000, seqlens=(3000, 0, 5, 1200))
+# longest row the selector holds in shared memory; longer rows stream their
+# keys from the score row on every pass
+SMEM_MAX_N = 40960
+VARLEN_LONG = _w("ragged", L=1, b=4, Hq=4, Hkv=1, n=140000, seqlens=(140000, 0, 5, 50000))
 
 SELECT_CASES = [
     # (name, workload, budget, alpha_key, policy, ban_mask, pool_k[, keep_last])
@@ -374,7 +378,7 @@ SELECT_CASES = [
     # the paper's other swept pool widths (Section 4: 3, 5, 7, 11, 15)
     ("combined_pool11", _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=5000), 0.10, 0.02, 0, 0, 11),
     ("varlen_global_pool11", VARLEN4, 0.20, 0.0, 1, 0, 11),
-    ("max_n", _w("long", L=1, b=1, Hq=4, Hkv=1, n=R.SELECT_MAX_N), 0.10, 0.0, 0, 0, 7),
+    ("max_n", _w("long", L=1, b=1, Hq=4, Hkv=1, n=SMEM_MAX_N), 0.10, 0.0, 0, 0, 7),
     # fair eviction (equal retention rate per role) and the recency floor
     ("fair_pool7", _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=5000), 0.10, 0.0, R.POLICY_FAIR, 0, 7),
     ("fair_no_key_varlen", VARLEN4, 0.20, 0.0, R.POLICY_FAIR, 1 << I.ROLE_KEY, 7),
@@ -382,22 +386,31 @@ SELECT_CASES = [
     ("floor32_global_varlen", VARLEN4, 0.10, 0.0, R.POLICY_GLOBAL, 0, 3, 32),
     ("floor_over_budget", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=3001), 0.05, 0.0, 0, 0, 7, 1000),
     ("floor_fair_mid_n", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=12001), 0.10, 0.0, R.POLICY_FAIR, 0, 7, 64),
-    ("floor_max_n", _w("long", L=1, b=1, Hq=4, Hkv=1, n=R.SELECT_MAX_N), 0.10, 0.0, 0, 0, 7, 64),
+    ("floor_max_n", _w("long", L=1, b=1, Hq=4, Hkv=1, n=SMEM_MAX_N), 0.10, 0.0, 0, 0, 7, 64),
     # role quotas with the slack of saturated buckets filled by score
     ("slack_b50", _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=5000), 0.50, 0.02, R.POLICY_SLACK, 0, 7),
     ("slack_b30_no_key_varlen", VARLEN4, 0.30, 0.0, R.POLICY_SLACK, 0, 7),
     ("slack_floor_mid_n", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=12001), 0.20, 0.02, R.POLICY_SLACK, 0, 7, 64),
-    ("slack_ban_max_n", _w("long", L=1, b=1, Hq=4, Hkv=1, n=R.SELECT_MAX_N), 0.30, 0.02, R.POLICY_SLACK,
+    ("slack_ban_max_n", _w("long", L=1, b=1, Hq=4, Hkv=1, n=SMEM_MAX_N), 0.30, 0.02, R.POLICY_SLACK,
      1 << I.ROLE_KEY, 1),
     # Algorithm 1's per-bucket ceilings taken literally (rows widened by
     # kept_extra = N_ROLES - 1 unless given), and widened rows under the exact split
     ("ceil_b10_pool7", _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=5000), 0.10, 0.02, R.POLICY_CEIL, 0, 7),
     ("ceil_varlen_floor32", VARLEN4, 0.05, 0.0, R.POLICY_CEIL, 0, 7, 32),
-    ("ceil_ban_max_n", _w("long", L=1, b=1, Hq=4, Hkv=1, n=R.SELECT_MAX_N), 0.30, 0.02, R.POLICY_CEIL,
+    ("ceil_ban_max_n", _w("long", L=1, b=1, Hq=4, Hkv=1, n=SMEM_MAX_N), 0.30, 0.02, R.POLICY_CEIL,
      1 << I.ROLE_KEY, 1),
     ("ceil_full_budget", _w("llama8b", L=1, b=1, Hq=4, Hkv=1, n=777), 1.0, 0.02, R.POLICY_CEIL, 0, 3),
     ("ceil_mid_n_extra9", _w("llama8b", L=1, b=1, Hq=8, Hkv=2, n=12001), 0.20, 0.02, R.POLICY_CEIL, 0, 7, 0, 9),
     ("quota_varlen_extra5", VARLEN4, 0.10, 0.02, 0, 0, 7, 0, 5),
+    # rows past the shared-memory maximum (streaming mode), up to the ABI limit
+    ("stream_65536", _w("long", L=1, b=1, Hq=4, Hkv=1, n=65536), 0.10, 0.02, 0, 0, 7),
+    ("stream_131072_global_pool5", _w("long", L=1, b=1, Hq=4, Hkv=1, n=131072), 0.10, 0.0, 1, 0, 5),
+    ("stream_131072_slack_floor", _w("long", L=1, b=1, Hq=4, Hkv=1, n=131072), 0.20, 0.02, R.POLICY_SLACK, 0,
+     7, 64),
+    ("stream_262144_ceil_pool3", _w("long", L=1, b=1, Hq=4, Hkv=1, n=R.SELECT_MAX_N), 0.05, 0.02,
+     R.POLICY_CEIL, 0, 3),
+    ("stream_varlen_fair", VARLEN_LONG, 0.10, 0.0, R.POLICY_FAIR, 1 << I.ROLE_KEY, 7),
+    ("stream_varlen_quota_floor", VARLEN_LONG, 0.30, 0.02, 0, 0, 11, 32),
 ]
 
 
@@ -449,6 +462,7 @@ def test_role_alloc_select_bit_exact(case):
 NARROW_CASES = [
     # (name, n, policy, pool_k, spread): page-constant scores in [2, 2 + spread)
     ("narrow_quota", 20000, 0, 1, 0.2),
+    ("narrow_global_stream", 70000, 1, 3, 0.2),
     ("narrow_global_pool7", 20000, 1, 7, 0.2),
     ("narrow_fair_short", 9000, 2, 1, 0.2),
     ("constant_global", 20000, 1, 1, 0.0),
@@ -519,11 +533,12 @@ def test_select_six_role_taxonomy(akey):
             assert per[0] == 0 and per[3] == 0
 
 
-@pytest.mark.parametrize("pool_k", [1, 7])
-def test_select_nan_scores_flagged_and_lowest(pool_k):
+@pytest.mark.parametrize("pool_k,n", [(1, 3001), (7, 3001), (5, 50001)])
+def test_select_nan_scores_flagged_and_lowest(pool_k, n):
     """A NaN score sets STATUS_NONFINITE; every pooled window holding a NaN
-    ranks below every other token (kept last, ties in index order)."""
-    w = _w("llama8b", L=1, b=2, Hq=4, Hkv=1, n=3001)
+    ranks below every other token (kept last, ties in index order); also in
+    the streaming mode (n above the shared-memory maximum)."""
+    w = _w("llama8b", L=1, b=2, Hq=4, Hkv=1, n=n)
     roles_np = I.workload_roles(w, 4)
     batch = lib_batch(w, DEV)
     g = torch.Generator().manual_seed(11)

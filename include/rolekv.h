@@ -80,6 +80,9 @@ extern "C" {
 #define ROLEKV_STATUS_NONFINITE 1   /* a NaN score was seen by the selector    */
 #define ROLEKV_STATUS_BAD_INDEX 2   /* kv_compact met an index >= the length  */
 #define ROLEKV_STATUS_TIMEOUT 4     /* a bounded device wait gave up          */
+#define ROLEKV_STATUS_BOUNDS 8      /* checked build: an access fell outside the
+                                       extent the call's shapes give its buffer
+                                       and was skipped                         */
 
 #define ROLEKV_POLICY_ROLE_QUOTA 0  /* the combined method (Section 4.1)       */
 #define ROLEKV_POLICY_GLOBAL 1      /* plain top-k, optional role ban (Sec. 4) */
@@ -366,6 +369,33 @@ int rolekv_selftest_wait(int64_t limit_ns, int32_t* status_dev, void* stream);
  * that one call.  It lets a caller check, without a fault, that the real
  * kernel's abort path reports the stuck wait and leaves the device usable. */
 int rolekv_selftest_score_timeout(int64_t limit_ns);
+
+/* Checked build (no counterpart in the paper).  The library can be built a
+ * second time with -DROLEKV_CHECKED (librolekv_checked.so beside
+ * librolekv.so, same entry points).  Every kernel there checks each global
+ * load or store whose address it computes from run-time data (kept indices,
+ * sequence offsets, unit and chunk offsets, strides) against the extent the
+ * call's shapes and strides give that buffer.  An access outside it is
+ * skipped and ROLEKV_STATUS_BOUNDS is OR-ed into the status word: a kernel
+ * bug then shows up as a status bit and a wrong output, not as a memory
+ * fault.  Loads and stores through TMA tensor maps are bounded by the maps
+ * themselves and are not checked again.  The checks cost time; the plain
+ * build has none.
+ *
+ * rolekv_checked_build() returns 1 in the checked build and 0 in the plain
+ * one. */
+int rolekv_checked_build(void);
+
+/* Diagnostic for the checked build (no counterpart in the paper): the next
+ * kv_compact call made on the calling thread takes its output extent as
+ * `rows` kept rows smaller than its shapes give (1 .. 1e6), so that the
+ * checks on the last rows fire although every access is inside the real
+ * buffer.  That call skips those rows' stores (their output is left as it
+ * was) and ORs ROLEKV_STATUS_BOUNDS into its status word.  The arming is used
+ * up by that one call.  It lets a caller see that the checks report and skip
+ * without provoking a single out-of-range access.  Returns
+ * ROLEKV_ERR_UNSUPPORTED in the plain build. */
+int rolekv_selftest_shrink_extent(int64_t rows);
 
 #ifdef __cplusplus
 }

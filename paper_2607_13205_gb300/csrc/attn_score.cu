@@ -402,12 +402,15 @@ __device__ __forceinline__ void rowstats_epilogue(const ScoreArgs& a, const Work
   }
   if (a.mode == kModeSnapKV) {
     const int64_t slot = static_cast<int64_t>(w.u) * a.n_chunks + w.chunk;
-    a.partials[slot * kRowsMax + row] = make_float2(m2, l);
-    if (nrt == 1) a.partials[slot * kRowsMax + 128 + row] = make_float2(-INFINITY, 0.f);
+    if (in_bounds(slot * kRowsMax + row, 1, a.ext_partials, a.status))
+      a.partials[slot * kRowsMax + row] = make_float2(m2, l);
+    if (nrt == 1 && in_bounds(slot * kRowsMax + 128 + row, 1, a.ext_partials, a.status))
+      a.partials[slot * kRowsMax + 128 + row] = make_float2(-INFINITY, 0.f);
   } else if (w.rb1 > w.rb0) {
     const int64_t o = (static_cast<int64_t>(w.u) * a.nrb_max + rb) * kRowsMax;
-    a.lse2[o + row] = (l > 0.f) ? -(m2 + __log2f(l)) : -INFINITY;
-    if (nrt == 1) a.lse2[o + 128 + row] = -INFINITY;
+    if (in_bounds(o + row, 1, a.ext_lse2, a.status))
+      a.lse2[o + row] = (l > 0.f) ? -(m2 + __log2f(l)) : -INFINITY;
+    if (nrt == 1 && in_bounds(o + 128 + row, 1, a.ext_lse2, a.status)) a.lse2[o + 128 + row] = -INFINITY;
   }
 }
 
@@ -493,7 +496,7 @@ __device__ __forceinline__ void colsum_epilogue(const ScoreArgs& a, const Work& 
 #pragma unroll
       for (int x = 1; x < kParts; ++x) total += sh.red[(x - 1) * kTileKeys + kl];
       mbar_arrive(sh.red_empty);
-      if (t < n) {
+      if (t < n && in_bounds(sbase + t, 1, a.ext_scores, a.status)) {
         if (a.mode == kModeH2O)
           atomicAdd(a.prepool + sbase + t, total);   // one query block's share
         else
@@ -1154,8 +1157,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           sh.merge[row] = make_float2(m2, l);      // (slot 0: the leader's own)
         } else {
           const int64_t slot = static_cast<int64_t>(u) * a.n_chunks + chunk;
-          a.partials[slot * kRowsMax + row] = make_float2(m2, l);
-          if (nrt == 1) a.partials[slot * kRowsMax + 128 + row] = make_float2(-INFINITY, 0.f);
+          if (in_bounds(slot * kRowsMax + row, 1, a.ext_partials, a.status))
+            a.partials[slot * kRowsMax + row] = make_float2(m2, l);
+          if (nrt == 1 && in_bounds(slot * kRowsMax + 128 + row, 1, a.ext_partials, a.status))
+            a.partials[slot * kRowsMax + 128 + row] = make_float2(-INFINITY, 0.f);
           __threadfence();
         }
       }
@@ -1199,13 +1204,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int64_t Hq = static_cast<int64_t>(a.Hkv) * a.G;
             const int64_t o = a.varlen ? (un.l * Hq + hq) * a.T + un.tok0 + p
                                        : ((static_cast<int64_t>(un.l) * a.b + un.s) * Hq + hq) * a.n_max + p;
-            nl = -__ldg(fa.h2o_lse + o) * kLog2e;
+            if (in_bounds(o, 1, fa.ext_h2o_lse, a.status)) nl = -__ldg(fa.h2o_lse + o) * kLog2e;
           }
         } else if (h2o) {
           const float2 ml = sh.merge[j];
           if (p >= 0 && ml.y > 0.f) nl = -(ml.x + log2f(ml.y));
         } else if (fa.single) {
-          nl = (p >= 0) ? a.lse2[static_cast<int64_t>(u) * kRowsMax + j] : -INFINITY;
+          const int64_t o = static_cast<int64_t>(u) * kRowsMax + j;
+          nl = (p >= 0 && in_bounds(o, 1, a.ext_lse2, a.status)) ? a.lse2[o] : -INFINITY;
         } else if (p >= 0) {
           // one online merge over the chunks, eight independent loads in flight
           const float2* part_j = a.partials + static_cast<int64_t>(u) * a.n_chunks * kRowsMax + j;
@@ -1214,8 +1220,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             float2 v[8];
 #pragma unroll
             for (int i = 0; i < 8; ++i)
-              v[i] = (c0 + i < a.n_chunks) ? __ldcg(&part_j[(c0 + i) * kRowsMax])
-                                           : make_float2(-INFINITY, 0.f);
+              v[i] = (c0 + i < a.n_chunks &&
+                      in_bounds(static_cast<int64_t>(u) * a.n_chunks * kRowsMax + j + (c0 + i) * kRowsMax, 1,
+                                a.ext_partials, a.status))
+                         ? __ldcg(&part_j[(c0 + i) * kRowsMax])
+                         : make_float2(-INFINITY, 0.f);
 #pragma unroll
             for (int i = 0; i < 8; ++i) {
               if (v[i].y > 0.f) {
@@ -1310,7 +1319,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!ok) break;
           const float total = colsum + sh.red[grp * kTileKeys + kl];
           mbar_arrive(&sh.red_empty[grp]);
-          if (t < n) {
+          if (t < n && in_bounds(sbase + t, 1, a.ext_scores, a.status)) {
             if (h2o)
               atomicAdd(a.prepool + sbase + t, total);   // one query block's share
             else
@@ -1347,22 +1356,26 @@ __global__ void snapkv_lse_kernel(const ScoreArgs a, const float* __restrict__ l
       const int64_t o =
           ((static_cast<int64_t>(un.l) * a.b + un.s) * (static_cast<int64_t>(a.Hkv) * a.G) +
            static_cast<int64_t>(un.h) * a.G + g) * a.W + i;
-      out = lse_win[o] * kLog2e;
+      if (in_bounds(o, 1, a.ext_lse_win, a.status)) out = lse_win[o] * kLog2e;
     } else {
-      const float2* part = a.partials + static_cast<int64_t>(u) * a.n_chunks * kRowsMax + j;
-      float m = -INFINITY;
-      for (int c = 0; c < a.n_chunks; ++c) m = fmaxf(m, part[c * kRowsMax].x);
-      if (m > -INFINITY) {
-        float l = 0.f;
-        for (int c = 0; c < a.n_chunks; ++c) {
-          const float2 v = part[c * kRowsMax];
-          if (v.y > 0.f) l += v.y * exp2f(v.x - m);
+      const int64_t p0 = static_cast<int64_t>(u) * a.n_chunks * kRowsMax + j;
+      const float2* part = a.partials + p0;
+      if (in_bounds(p0, static_cast<int64_t>(a.n_chunks - 1) * kRowsMax + 1, a.ext_partials, a.status)) {
+        float m = -INFINITY;
+        for (int c = 0; c < a.n_chunks; ++c) m = fmaxf(m, part[c * kRowsMax].x);
+        if (m > -INFINITY) {
+          float l = 0.f;
+          for (int c = 0; c < a.n_chunks; ++c) {
+            const float2 v = part[c * kRowsMax];
+            if (v.y > 0.f) l += v.y * exp2f(v.x - m);
+          }
+          out = m + log2f(l);
         }
-        out = m + log2f(l);
       }
     }
   }
-  a.lse2[static_cast<int64_t>(u) * kRowsMax + j] = -out;
+  if (in_bounds(static_cast<int64_t>(u) * kRowsMax + j, 1, a.ext_lse2, a.status))
+    a.lse2[static_cast<int64_t>(u) * kRowsMax + j] = -out;
 }
 
 // Stride-1 max-pool over each unit's score row, truncated at the sequence
@@ -1376,6 +1389,7 @@ __global__ void maxpool_kernel(const ScoreArgs a, const float* __restrict__ in,
   const int h = pool_k / 2;
   for (int t = part * blockDim.x + threadIdx.x; t < un.n; t += blocks_per_unit * blockDim.x) {
     const int lo = max(0, t - h), hi = min(un.n - 1, t + h);
+    if (!in_bounds(base + lo, hi - lo + 1, a.ext_scores, a.status)) continue;
     float m = in[base + lo];
     for (int x = lo + 1; x <= hi; ++x) m = fmaxf(m, in[base + x]);
     out[base + t] = m;

@@ -8,6 +8,7 @@
 
 #include <cstdint>
 
+#include "device_common.cuh"
 #include "internal.h"
 
 namespace rolekv {
@@ -69,14 +70,18 @@ __global__ void __launch_bounds__(kThreads) compact_kernel(const CompactArgs a, 
   const int j_end = static_cast<int>(K_s < j_begin + kRowsPerBlock ? K_s : j_begin + kRowsPerBlock);
   for (int j = j_begin + threadIdx.x / lanes_per_row; j < j_end; j += rows_per_pass) {
     const int64_t slot = kbase + j;
+    if (!in_bounds(slot, 1, a.ext_keep, a.status)) continue;
     const int32_t idx = a.keep_idx[slot];
     uint4 kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
     if (idx >= 0 && idx < n) {
-      kv = load_nc(reinterpret_cast<const uint4*>(a.k + kb + idx * a.k_tok) + piece);
-      vv = load_nc(reinterpret_cast<const uint4*>(a.v + vb + idx * a.v_tok) + piece);
+      if (in_bounds(kb + idx * a.k_tok + piece * 8, 8, a.ext_k, a.status))
+        kv = load_nc(reinterpret_cast<const uint4*>(a.k + kb + idx * a.k_tok) + piece);
+      if (in_bounds(vb + idx * a.v_tok + piece * 8, 8, a.ext_v, a.status))
+        vv = load_nc(reinterpret_cast<const uint4*>(a.v + vb + idx * a.v_tok) + piece);
     } else if (idx >= n && a.status != nullptr && piece == 0) {
       atomicOr(a.status, ROLEKV_STATUS_BAD_INDEX);
     }
+    if (!in_bounds(slot, 1, a.ext_out_rows, a.status)) continue;
     store_cs(reinterpret_cast<uint4*>(a.k_out + slot * a.d) + piece, kv);
     store_cs(reinterpret_cast<uint4*>(a.v_out + slot * a.d) + piece, vv);
   }

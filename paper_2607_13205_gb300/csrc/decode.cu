@@ -122,6 +122,25 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const Decod
   const int64_t vb = l * a.v_layer + (a.varlen ? row0 * a.v_tok : s * a.v_seq) + h * a.v_head;
   uint8_t* ks = stage_mem;
   uint8_t* vs = stage_mem + kStages * kStageRows * KSTR;
+#ifdef ROLEKV_CHECKED
+  // Checked build: this split's K and V rows, kept indices, the group's
+  // queries and its partials lie inside the extents the call's shapes give,
+  // or the CTA returns before any copy is issued.
+  {
+    const int64_t i0 = a.varlen ? (static_cast<int64_t>(l) * a.Hkv + h) * a.Ktot + row0
+                                : static_cast<int64_t>(u) * a.K_dense;
+    const int64_t q0 = l * a.q_layer + s * a.q_seq + static_cast<int64_t>(h) * G * a.q_head;
+    const int64_t p0 = (static_cast<int64_t>(u) * a.n_splits + split) * G * (a.d + 2);
+    if (!(in_bounds(kb + r0 * a.k_tok, (r1 - r0 - 1) * a.k_tok + a.d, a.ext_k, nullptr) &&
+          in_bounds(vb + r0 * a.v_tok, (r1 - r0 - 1) * a.v_tok + a.d, a.ext_v, nullptr) &&
+          (a.keep_idx == nullptr || in_bounds(i0 + r0, r1 - r0, a.ext_keep, nullptr)) &&
+          in_bounds(q0, (G - 1) * a.q_head + a.d, a.ext_q, nullptr) &&
+          in_bounds(p0, static_cast<int64_t>(G) * (a.d + 2), a.ext_part, nullptr))) {
+      if (threadIdx.x == 0 && a.status != nullptr) atomicOr(a.status, ROLEKV_STATUS_BOUNDS);
+      return;
+    }
+  }
+#endif
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < kStages; ++i) {
@@ -370,6 +389,10 @@ __global__ void __launch_bounds__(256) decode_combine_kernel(const DecodeArgs a)
   const int ns = (m + a.rows_per_split - 1) / a.rows_per_split;
   const float* base = a.part + (static_cast<int64_t>(u) * a.n_splits * a.G + g) * (a.d + 2);
   const int64_t stride = static_cast<int64_t>(a.G) * (a.d + 2);
+  const int64_t dst0 = l * a.o_layer + s * a.o_seq + static_cast<int64_t>(h * a.G + g) * a.o_head;
+  if (!in_bounds(base - a.part, (ns > 0 ? (ns - 1) * stride : 0) + a.d + 2, a.ext_part, a.status) ||
+      !in_bounds(dst0, a.d, a.ext_out, a.status))
+    return;                                          // (checked build only)
   float M = -INFINITY;
   for (int x = 0; x < ns; ++x) M = fmaxf(M, base[x * stride + a.d]);
   float L = 0.f, o[DPL];

@@ -241,6 +241,20 @@ __device__ __forceinline__ void tmem_reg_fence(uint32_t* r) {
 
 // ------------------------------------------------------------------ misc ----
 
+// Checked build: is the element range [i, i + len) inside a buffer of n
+// elements?  If not, ROLEKV_STATUS_BOUNDS is OR-ed into *status (may be
+// null) and the caller skips the access.  The plain build compiles every
+// check away.
+#ifdef ROLEKV_CHECKED
+__device__ __forceinline__ bool in_bounds(int64_t i, int64_t len, int64_t n, int32_t* status) {
+  if (i >= 0 && len >= 0 && i + len <= n) return true;
+  if (status != nullptr) atomicOr(status, ROLEKV_STATUS_BOUNDS);
+  return false;
+}
+#else
+__device__ __forceinline__ constexpr bool in_bounds(int64_t, int64_t, int64_t, int32_t*) { return true; }
+#endif
+
 __device__ __forceinline__ float fast_exp2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));

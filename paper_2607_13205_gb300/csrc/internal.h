@@ -38,6 +38,11 @@ struct ScoreArgs {
   float* lse2;                      // [unit][query block][256] log2-domain normalisers
   float* prepool;                   // score output before pooling
   int32_t* status;
+  // element extents the call's shapes give these buffers (checked build)
+  int64_t ext_scores;               // prepool and the pooled scores
+  int64_t ext_partials;
+  int64_t ext_lse2;
+  int64_t ext_lse_win;              // a caller-supplied window LSE
 };
 
 cudaError_t launch_attn_pass(int pass, int d, const CUtensorMap& kmap, const CUtensorMap& qmap,
@@ -59,6 +64,7 @@ struct FusedArgs {
   uint64_t wait_ns;                 // limit of the per-unit meeting point's wait
   int32_t hold;                     // arrivals the meeting point waits for beyond the
                                     // unit's chunks (0; 1 only in the timeout self-test)
+  int64_t ext_h2o_lse;              // elements of h2o_lse (checked build)
 };
 
 cudaError_t launch_snapkv_fused(int d, const CUtensorMap& kmap, const CUtensorMap& qmap,
@@ -91,6 +97,8 @@ struct SelectArgs {
   uint8_t* keep_mask;
   int32_t* kept_per_role;
   int32_t* status;
+  // element extents (checked build): scores and keep_mask, roles, keep_idx
+  int64_t ext_scores, ext_roles, ext_keep;
 };
 
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t stream);
@@ -110,6 +118,9 @@ struct QuestArgs {
   const uint16_t* k;
   int64_t k_layer, k_seq, k_head, k_tok;
   float* scores;
+  // element extents (checked build); quest_score has no status word, so an
+  // access outside them is skipped without a report
+  int64_t ext_scores, ext_q, ext_k;
 };
 
 cudaError_t launch_quest(const QuestArgs& a, cudaStream_t stream);
@@ -139,6 +150,8 @@ struct DecodeArgs {
   float* out;                       // fp32 outputs
   int64_t o_layer, o_seq, o_head;
   int32_t* status;
+  // element extents (checked build)
+  int64_t ext_q, ext_k, ext_v, ext_keep, ext_part, ext_out;
 };
 
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
@@ -164,6 +177,8 @@ struct CompactArgs {
   uint16_t* k_out;
   uint16_t* v_out;
   int32_t* status;
+  // element extents (checked build): K, V, kept slots, output rows
+  int64_t ext_k, ext_v, ext_keep, ext_out_rows;
 };
 
 cudaError_t launch_compact(const CompactArgs& a, cudaStream_t stream);

@@ -14,6 +14,7 @@
 
 #include <cstdint>
 
+#include "device_common.cuh"
 #include "internal.h"
 
 namespace rolekv {
@@ -72,6 +73,21 @@ __global__ void __launch_bounds__(kThreads, 3) quest_kernel(const QuestArgs a, i
   const int p_end = npages - p_begin < kPagesPerCta ? npages : p_begin + kPagesPerCta;
   const int d = a.d;
   const int CR = d / 8;                            // 16-byte chunks per row
+#ifdef ROLEKV_CHECKED
+  // Checked build: the unit's window queries, key rows and score row lie
+  // inside the extents the call's shapes give, or the CTA returns (quest_score
+  // has no status word to report it in).
+  {
+    const int w_eff = a.W < n ? a.W : n;
+    const int64_t q0 = l * a.q_layer + s * a.q_seq + static_cast<int64_t>(h) * a.G * a.q_head;
+    const int64_t k0 = l * a.k_layer + (a.varlen ? tok0 * a.k_tok : s * a.k_seq) + h * a.k_head;
+    const int64_t s0 =
+        a.varlen ? (static_cast<int64_t>(l) * a.Hkv + h) * a.T + tok0 : static_cast<int64_t>(u) * a.n_max;
+    if (!(w_eff == 0 || in_bounds(q0, (a.G - 1) * a.q_head + (w_eff - 1) * a.q_tok + d, a.ext_q, nullptr)) ||
+        !in_bounds(k0, (n - 1) * a.k_tok + d, a.ext_k, nullptr) || !in_bounds(s0, n, a.ext_scores, nullptr))
+      return;                                      // (uniform)
+  }
+#endif
 
   // ---- mean of the window rows (the last W_eff positions of the G heads):
   // thread (row group rg, chunk c) sums chunk c of rows rg, rg + RG, ...

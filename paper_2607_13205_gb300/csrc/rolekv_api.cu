@@ -12,6 +12,8 @@
 #include <cstring>
 #include <mutex>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "internal.h"
 #include "rolekv.h"
 
@@ -36,6 +38,17 @@ void stage_begin() { g_stage_cursor = 0; }
 // one arrival more than there are chunks, with this limit.
 thread_local bool g_timeout_test_armed = false;
 thread_local uint64_t g_timeout_test_ns = 0;
+// Checked-build self-test: rows the next kv_compact takes off its output extent.
+thread_local int64_t g_shrink_rows = 0;
+
+// An NVTX range over one library call, so that a profiler's timeline shows
+// each call, and the kernels it launches, under the call's name.
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 // Records the next stage event (if any) after a kernel launch.
 void stage_mark(cudaStream_t stream) {
@@ -285,6 +298,8 @@ int bind_workspace(ScorePlan& p, void* ws, size_t ws_bytes) {
   uint8_t* base = static_cast<uint8_t*>(ws);
   p.a.partials = reinterpret_cast<float2*>(base + p.off_partials);
   p.a.lse2 = reinterpret_cast<float*>(base + p.off_lse);
+  p.a.ext_partials = static_cast<int64_t>((p.off_lse - p.off_partials) / sizeof(float2));
+  p.a.ext_lse2 = static_cast<int64_t>((p.off_prepool - p.off_lse) / sizeof(float));
   p.work = p.fused ? reinterpret_cast<int32_t*>(base + p.off_work) : nullptr;
   return ROLEKV_OK;
 }
@@ -298,6 +313,8 @@ int run_snapkv(const BatchInfo& bi, const int32_t* cu_seqlens, const rolekv_tens
   set_strides(a, k, q_win);
   a.c1 = (scale > 0.f ? scale : 1.0f / std::sqrt(static_cast<float>(bi.d))) * 1.4426950408889634f;
   a.prepool = prepool;
+  a.ext_scores = score_elems(bi);
+  a.ext_lse_win = static_cast<int64_t>(bi.L) * bi.b * bi.Hq * W;
   a.status = status;
   a.cu_seqlens = cu_seqlens;
   CUtensorMap kmap, qmap;
@@ -382,6 +399,11 @@ void fill_compact(const BatchInfo& bi, const int32_t* cu_seqlens, int64_t budget
   a->k_out = static_cast<uint16_t*>(k_out);
   a->v_out = static_cast<uint16_t*>(v_out);
   a->status = status;
+  const int64_t rows = bi.varlen ? bi.T : bi.n_max;
+  a->ext_k = tensor_span(k, bi.L, bi.b, bi.Hkv, rows, bi.d, bi.varlen);
+  a->ext_v = tensor_span(v, bi.L, bi.b, bi.Hkv, rows, bi.d, bi.varlen);
+  a->ext_keep = bi.varlen ? static_cast<int64_t>(bi.L) * bi.Hkv * a->Ktot : bi.n_units * a->K_dense;
+  a->ext_out_rows = a->ext_keep;
 }
 
 int check_compact_args(const BatchInfo& bi, const rolekv_tensor& k, const rolekv_tensor& v,
@@ -452,6 +474,9 @@ int fill_select(const BatchInfo& bi, const rolekv_batch* bt, const rolekv_select
   a->Ktot = 0;
   if (bi.varlen)
     for (int s = 0; s < bi.b; ++s) a->Ktot += kept_rows(bt->seqlens_host[s], a->budget_fx, bi.kept_extra);
+  a->ext_scores = score_elems(bi);
+  a->ext_roles = bi.varlen ? bi.T : static_cast<int64_t>(bi.b) * bi.n_max;
+  a->ext_keep = bi.varlen ? static_cast<int64_t>(bi.L) * bi.Hkv * a->Ktot : bi.n_units * a->K_dense;
   return ROLEKV_OK;
 }
 
@@ -545,6 +570,7 @@ int snapkv_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k
                  int32_t pool_k, float scale, const float* lse_win, float* scores,
                  float* scores_prepool, void* workspace, size_t workspace_bytes,
                  int32_t* status_dev, void* stream) {
+  NvtxRange nvtx("rolekv:snapkv_score");
   BatchInfo bi;
   int rc = check_batch(batch, &bi);
   if (rc) return rc;
@@ -578,6 +604,7 @@ int snapkv_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k
 int h2o_score(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k, float scale,
               const float* lse, float* scores, void* workspace, size_t workspace_bytes,
               int32_t* status_dev, void* stream) {
+  NvtxRange nvtx("rolekv:h2o_score");
   BatchInfo bi;
   int rc = check_batch(batch, &bi);
   if (rc) return rc;
@@ -597,6 +624,7 @@ int h2o_score(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k, float
   a.c1 = (scale > 0.f ? scale : 1.0f / std::sqrt(static_cast<float>(bi.d))) * 1.4426950408889634f;
   a.prepool = scores;
   a.status = status_dev;
+  a.ext_scores = score_elems(bi);
   CUtensorMap kmap, qmap;
   const int64_t rows = bi.varlen ? bi.T : bi.n_max;
   rc = make_row_map(&kmap, k, tensor_span(k, bi.L, bi.b, bi.Hkv, rows, bi.d, bi.varlen), kTileKeys);
@@ -616,6 +644,7 @@ int h2o_score(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k, float
   fa.n_items = p.n_items;
   fa.single = lse != nullptr;
   fa.h2o_lse = lse;
+  fa.ext_h2o_lse = static_cast<int64_t>(bi.L) * bi.Hq * (bi.varlen ? bi.T : static_cast<int64_t>(bi.b) * bi.n_max);
   fa.wait_ns = kWaitLimitNs;
   e = launch_snapkv_fused(bi.d, kmap, qmap, fa, st);
   if (e != cudaSuccess) return cuda_fail(e, "h2o fused score");
@@ -625,6 +654,7 @@ int h2o_score(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k, float
 
 int quest_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k, int32_t W,
                 int32_t page, float* scores, void* stream) {
+  NvtxRange nvtx("rolekv:quest_score");
   BatchInfo bi;
   int rc = check_batch(batch, &bi);
   if (rc) return rc;
@@ -663,6 +693,9 @@ int quest_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k,
   a.k_head = k.s_head;
   a.k_tok = k.s_tok;
   a.scores = scores;
+  a.ext_scores = score_elems(bi);
+  a.ext_q = tensor_span(q_win, bi.L, bi.b, bi.Hq, W, bi.d, false);
+  a.ext_k = tensor_span(k, bi.L, bi.b, bi.Hkv, bi.varlen ? bi.T : bi.n_max, bi.d, bi.varlen);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   stage_begin();
   cudaError_t e = launch_quest(a, st);
@@ -675,6 +708,7 @@ int role_alloc_select(const rolekv_batch* batch, const float* scores, const uint
                       const rolekv_select_params* params, int32_t pool_k, int32_t* keep_idx,
                       uint8_t* keep_mask, int32_t* kept_per_role, int32_t* status_dev,
                       void* stream) {
+  NvtxRange nvtx("rolekv:role_alloc_select");
   BatchInfo bi;
   int rc = check_batch(batch, &bi);
   if (rc) return rc;
@@ -756,6 +790,7 @@ int decode_attention(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k
                      rolekv_tensor v_cache, const int32_t* keep_idx, float budget, float scale,
                      float* out, void* workspace, size_t workspace_bytes, int32_t* status_dev,
                      void* stream) {
+  NvtxRange nvtx("rolekv:decode_attention");
   BatchInfo bi;
   int rc = check_batch(batch, &bi);
   if (rc) return rc;
@@ -819,6 +854,15 @@ int decode_attention(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k
   a.o_layer = a.o_seq * bi.b;
   a.o_head = bi.d;
   a.status = status_dev;
+  {
+    const int64_t rows = bi.varlen ? total : m_max;   // cache rows per (layer, head) / unit
+    a.ext_q = tensor_span(q, bi.L, bi.b, bi.Hq, 1, bi.d, false);
+    a.ext_k = tensor_span(k_cache, bi.L, bi.b, bi.Hkv, rows, bi.d, bi.varlen);
+    a.ext_v = tensor_span(v_cache, bi.L, bi.b, bi.Hkv, rows, bi.d, bi.varlen);
+    a.ext_keep = keep_idx == nullptr ? 0 : static_cast<int64_t>(bi.L) * bi.Hkv * (bi.varlen ? total : bi.b * m_max);
+    a.ext_part = static_cast<int64_t>(workspace_bytes / sizeof(float));
+    a.ext_out = static_cast<int64_t>(bi.L) * bi.b * bi.Hq * bi.d;
+  }
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   stage_begin();
   cudaError_t e = launch_decode(a, st);
@@ -830,6 +874,7 @@ int decode_attention(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k
 int kv_compact(const rolekv_batch* batch, rolekv_tensor k, rolekv_tensor v,
                const int32_t* keep_idx, float budget, void* k_out, void* v_out,
                int32_t* status_dev, void* stream) {
+  NvtxRange nvtx("rolekv:kv_compact");
   BatchInfo bi;
   int rc = check_batch(batch, &bi);
   if (rc) return rc;
@@ -840,6 +885,10 @@ int kv_compact(const rolekv_batch* batch, rolekv_tensor k, rolekv_tensor v,
   CompactArgs a;
   fill_compact(bi, batch->cu_seqlens_dev, to_fixed(budget), batch->seqlens_host, k, v, keep_idx,
                k_out, v_out, status_dev, &a);
+  if (g_shrink_rows > 0) {                         // (checked-build self-test only)
+    a.ext_out_rows -= g_shrink_rows;
+    g_shrink_rows = 0;
+  }
   if (bi.n_max == 0) return ROLEKV_OK;
   stage_begin();
   cudaError_t e = launch_compact(a, static_cast<cudaStream_t>(stream));
@@ -854,6 +903,7 @@ int rolekv_compress(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tenso
                     const rolekv_select_params* params, int32_t* keep_idx, void* k_out,
                     void* v_out, int32_t* kept_per_role, void* workspace,
                     size_t workspace_bytes, int32_t* status_dev, void* stream) {
+  NvtxRange nvtx("rolekv:rolekv_compress");
   BatchInfo bi;
   int rc = check_batch(batch, &bi);
   if (rc) return rc;
@@ -906,6 +956,7 @@ int snapkv_score_noalloc(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_
                          int32_t W, int32_t pool_k, float scale, const float* lse_win,
                          float* scores, float* scores_prepool, int32_t* status_dev,
                          void* stream) {
+  NvtxRange nvtx("rolekv:snapkv_score_noalloc");
   BatchInfo bi;
   int rc = check_batch(batch, &bi);
   if (rc) return rc;
@@ -948,6 +999,26 @@ int snapkv_score_noalloc(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_
   if (e != cudaSuccess) return cuda_fail(e, "max-pool");
   stage_mark(st);
   return ROLEKV_OK;
+}
+
+int rolekv_checked_build(void) {
+#ifdef ROLEKV_CHECKED
+  return 1;
+#else
+  return 0;
+#endif
+}
+
+int rolekv_selftest_shrink_extent(int64_t rows) {
+#ifdef ROLEKV_CHECKED
+  if (rows < 1 || rows > 1000000)
+    return fail(ROLEKV_ERR_INVALID_ARG, "rows=%lld outside 1..1e6", static_cast<long long>(rows));
+  g_shrink_rows = rows;
+  return ROLEKV_OK;
+#else
+  (void)rows;
+  return fail(ROLEKV_ERR_UNSUPPORTED, "not a checked build (librolekv_checked.so has the checks)");
+#endif
 }
 
 int rolekv_selftest_score_timeout(int64_t limit_ns) {

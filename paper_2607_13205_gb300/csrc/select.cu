@@ -692,6 +692,21 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
     }
   }
 
+  // Checked build: the unit's score row (and mask row), role row, kept row
+  // and per-role counts lie inside the extents the call's shapes give, or the
+  // whole unit is skipped.
+#ifdef ROLEKV_CHECKED
+  __syncthreads();
+  if (!(in_bounds(sbase, n, a.ext_scores, nullptr) && in_bounds(rbase, n, a.ext_roles, nullptr) &&
+        in_bounds(S.keep_off, width, a.ext_keep, nullptr) &&
+        (a.kept_per_role == nullptr ||
+         in_bounds(static_cast<int64_t>(u) * a.n_roles, a.n_roles, static_cast<int64_t>(a.n_units) * a.n_roles,
+                   nullptr)))) {
+    if (tid == 0 && a.status != nullptr) atomicOr(a.status, ROLEKV_STATUS_BOUNDS);
+    return;
+  }
+#endif
+
   // ---- pass 1: load, pool, key, first-digit histograms
   {
     bool nan_hint = false;
@@ -1146,7 +1161,8 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
     while (m != 0) {
       const int t = q * 32 + (__ffs(m) - 1) - off;
       m &= m - 1;
-      dst[pos++] = t;
+      if (in_bounds(pos, 1, width, a.status)) dst[pos] = t;   // (the unit's own row)
+      ++pos;
       if (count_roles) kr += shl64(1ull, 8u * __ldg(v.rp + t));
     }
   }, S.warp_tot);

@@ -14,10 +14,14 @@ from typing import Optional, Sequence
 
 import torch
 
-_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "librolekv.so")
+# ROLEKV_CHECKED=1 in the environment selects the checked build (every
+# computed global access checked against its buffer's extent; a miss sets
+# STATUS_BOUNDS and is skipped), which has the same entry points.
+_LIB_NAME = "librolekv_checked.so" if os.environ.get("ROLEKV_CHECKED") == "1" else "librolekv.so"
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), _LIB_NAME)
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_CUDA = 0, 1, 2, 3, 4
-STATUS_NONFINITE, STATUS_BAD_INDEX, STATUS_TIMEOUT = 1, 2, 4
+STATUS_NONFINITE, STATUS_BAD_INDEX, STATUS_TIMEOUT, STATUS_BOUNDS = 1, 2, 4, 8
 POLICY_ROLE_QUOTA, POLICY_GLOBAL, POLICY_FAIR, POLICY_SLACK, POLICY_CEIL = 0, 1, 2, 3, 4
 MAX_ROLES = 8
 SELECT_MAX_N = 262144
@@ -78,6 +82,8 @@ _SIGNATURES = [
      [ctypes.POINTER(BatchDesc), Tensor, Tensor, ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p,
       ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p, ctypes.c_void_p]),
     ("rolekv_selftest_score_timeout", ctypes.c_int, [ctypes.c_int64]),
+    ("rolekv_checked_build", ctypes.c_int, []),
+    ("rolekv_selftest_shrink_extent", ctypes.c_int, [ctypes.c_int64]),
     ("role_alloc_select", ctypes.c_int,
      [ctypes.POINTER(BatchDesc), ctypes.c_void_p, ctypes.c_void_p, ctypes.POINTER(SelectParams),
       ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
@@ -310,6 +316,18 @@ def selftest_score_timeout(limit_ns: int) -> None:
     """Arm the next two-pass SnapKV score on this thread to time out at its
     per-unit meeting point after limit_ns (diagnostic; see rolekv.h)."""
     _check(lib().rolekv_selftest_score_timeout(int(limit_ns)))
+
+
+def checked_build() -> bool:
+    """Whether the loaded library is the checked build."""
+    return lib().rolekv_checked_build() == 1
+
+
+def selftest_shrink_extent(rows: int) -> None:
+    """Checked build only: the next kv_compact on this thread takes its output
+    extent as `rows` rows smaller, so its checks on the last rows fire
+    (diagnostic; see rolekv.h)."""
+    _check(lib().rolekv_selftest_shrink_extent(int(rows)))
 
 
 def role_alloc_select(batch: Batch, scores: torch.Tensor, roles: torch.Tensor, params: SelectParams,

@@ -44,6 +44,23 @@ def test_every_declared_symbol_is_exported(lib):
         assert hasattr(lib, n), f"{n} declared in rolekv.h but not exported"
 
 
+def test_checked_build_loads_and_exports_every_symbol(lib):
+    """The checked library (-DROLEKV_CHECKED) is built beside the plain one,
+    exports the same entry points and says which it is; its extent self-test
+    is refused by the plain build.  Host calls only."""
+    if not os.path.exists(B.CHECKED_LIB_PATH):
+        B.build(checked=True)
+    chk = ctypes.CDLL(B.CHECKED_LIB_PATH)
+    for n in _declared_functions():
+        assert hasattr(chk, n), f"{n} declared in rolekv.h but not exported by the checked build"
+    assert chk.rolekv_checked_build() == 1
+    assert lib.rolekv_checked_build() == 0
+    shrink = chk.rolekv_selftest_shrink_extent
+    shrink.argtypes = [ctypes.c_int64]
+    assert shrink(0) == R.ERR_INVALID_ARG          # (an out-of-range count arms nothing)
+    assert lib.rolekv_selftest_shrink_extent(1) == R.ERR_UNSUPPORTED
+
+
 def test_kept_count_matches_oracle(lib):
     for n in (0, 1, 7, 100, 2048, 8192, 32768, 40960, 123457):
         for b in (0.05, 0.1, 0.2, 0.3, 0.5, 0.75, 1.0, 0.333):

@@ -146,9 +146,9 @@ TRAFFIC_FILE = os.path.join(ROOT, "profiles", "dram_traffic.md")
 KERNEL_SOURCES = {
     ("snapkv", "score"): ["attn_score.cu", "device_common.cuh", "internal.h"],
     ("h2o", "score"): ["attn_score.cu", "device_common.cuh", "internal.h"],
-    ("quest", "score"): ["quest.cu", "internal.h"],
-    ("snapkv", "select"): ["select.cu", "internal.h"],
-    ("snapkv", "compact"): ["compact.cu", "internal.h"],
+    ("quest", "score"): ["quest.cu", "device_common.cuh", "internal.h"],
+    ("snapkv", "select"): ["select.cu", "device_common.cuh", "internal.h"],
+    ("snapkv", "compact"): ["compact.cu", "device_common.cuh", "internal.h"],
 }
 
 

@@ -31,6 +31,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdint>
 #include <type_traits>
@@ -1441,7 +1442,10 @@ static cudaError_t launch_fused(const CUtensorMap& kmap, const CUtensorMap& qmap
   // of a unit's chunks in the same round.
   const int nc = a.s.n_chunks;
   if (nc < 1 || nc > sms) return cudaErrorInvalidConfiguration;
-  const int grid = (sms / nc) * nc;
+  // (no more CTAs than items: a small batch does not set up idle CTAs; the
+  // count stays a multiple of the chunks per unit)
+  const int items = ((a.n_items + nc - 1) / nc) * nc;
+  const int grid = std::min((sms / nc) * nc, std::max(items, nc));
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(grid));
   cfg.blockDim = dim3(kThreads);

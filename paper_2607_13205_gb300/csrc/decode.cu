@@ -6,9 +6,13 @@
 // are skipped; with budget 1 and no index the full cache).  Memory-bound: the
 // cache rows are read once.  Split-K: CTA (unit, split) takes up to 1024 rows
 // (a unit's splits equal in length).  A producer warp streams them into two
-// shared-memory stages of 64 K rows and 64 V rows with bulk copies (K one
-// copy per row, into rows padded by 16 bytes; V one copy per stage when the
-// rows are contiguous).  Each of four consumer warps takes 16 rows of a stage:
+// shared-memory stages of 64 K rows and 64 V rows.  K goes through a tensor
+// map, one copy per 64-column half of a stage, 128-byte swizzled so that the
+// consumers' fragment loads stay conflict-free; V goes in one copy per stage
+// (a bulk copy when the rows are contiguous, a tensor-map copy when they are
+// strided, as in a packed varlen cache).  Layouts a tensor map cannot
+// describe fall back to one bulk copy per row (K rows padded by 16 bytes).
+// Each of four consumer warps takes 16 rows of a stage:
 // the G x 16 dot products are one m16n8k16 bf16 MMA tile per 16 dimensions
 // (cache rows x query heads padded to 8, fp32 accumulate), so no cross-lane
 // reduction is needed; the online softmax (log2 units) runs in that fragment
@@ -65,6 +69,13 @@ __host__ __device__ constexpr int k_stride_bytes(int d) { return 2 * d + 16; }
 __host__ __device__ constexpr int decode_smem_bytes(int d) {
   return kStages * kStageRows * (k_stride_bytes(d) + 2 * d);
 }
+// With K through a tensor map (KT): a stage's K rows in 64-column halves of
+// kStageRows x 128 bytes each, 128-byte swizzled (the 16-byte chunk index of
+// row r XOR-ed with r mod 8), which keeps the fragment loads conflict-free
+// without padding; 1 KB of room to align the stages to the swizzle's 1 KB.
+__host__ __device__ constexpr int decode_smem_bytes_kt(int d) {
+  return kStages * kStageRows * (2 * d + 2 * d) + 1024;
+}
 
 __device__ __forceinline__ uint32_t lds32(const uint8_t* p) { return *reinterpret_cast<const uint32_t*>(p); }
 
@@ -84,13 +95,18 @@ __device__ __forceinline__ void mma16816(float* c, uint32_t a0, uint32_t a1, uin
 // and 2t + 1); the online softmax runs there; the probabilities and rescale
 // factors then go through a small per-warp shared buffer to the output
 // accumulation, where the lanes run over the head dimension (DPL each).
-template <int DPL, int GM>
-__global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const DecodeArgs a) {
+template <int DPL, int GM, bool KT>
+__global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const DecodeArgs a,
+                                                                     const __grid_constant__ CUtensorMap k_map,
+                                                                     const __grid_constant__ CUtensorMap v_map) {
   constexpr int D = DPL * 32;
   constexpr int KS = D / 16;                                // MMA k-steps
-  constexpr int KSTR = k_stride_bytes(D);
+  constexpr int KSTR = KT ? 2 * D : k_stride_bytes(D);      // bytes of K per row in a stage
   constexpr int VSTR = 2 * D;
-  extern __shared__ __align__(128) uint8_t stage_mem[];     // K stages, then V stages
+  constexpr int KHALF = kStageRows * 128;                   // KT: one 64-column half of a stage
+  extern __shared__ __align__(128) uint8_t stage_raw[];     // K stages, then V stages
+  uint8_t* stage_mem = KT ? stage_raw + ((1024u - (static_cast<uint32_t>(__cvta_generic_to_shared(stage_raw)) & 1023u)) & 1023u)
+                          : stage_raw;
   __shared__ uint64_t full_bar[kStages], empty_bar[kStages];
   __shared__ int abort_flag;
   __shared__ float red[kDecWarps][GM][2];                   // per-warp (max2, sum) per head
@@ -173,13 +189,35 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const Decod
       if (!__shfl_sync(0xffffffffu, static_cast<int>(ok), 0)) break;
       const int rs = r0 + st * kStageRows;
       const int nr = (r1 - rs < kStageRows) ? r1 - rs : kStageRows;
-      if (lane == 0) mbar_arrive_expect_tx(&full_bar[slot], static_cast<uint32_t>(2 * nr * VSTR));
+      // (strided V rows: one tensor-map copy of the whole stage, kStageRows
+      // rows whatever nr is -- the rows past the unit are not used)
+      const uint32_t vbytes = static_cast<uint32_t>((a.v_tma ? kStageRows : nr) * VSTR);
+      const uint32_t kbytes = static_cast<uint32_t>((KT ? kStageRows : nr) * VSTR);
+      if (lane == 0) mbar_arrive_expect_tx(&full_bar[slot], kbytes + vbytes);
       __syncwarp();
       uint8_t* kd = ks + slot * kStageRows * KSTR;
       uint8_t* vd = vs + slot * kStageRows * VSTR;
-      for (int r = lane; r < nr; r += 32)
-        bulk_copy_g2s(kd + r * KSTR, a.k + kb + static_cast<int64_t>(rs + r) * a.k_tok, VSTR, &full_bar[slot]);
-      if (vc) {
+      if constexpr (KT) {
+        // the whole stage, one tensor-map copy per 64-column half (the rows
+        // past the unit are not used)
+        if (lane == 0) {
+          const int64_t e0 = kb + static_cast<int64_t>(rs) * a.k_tok;
+#pragma unroll
+          for (int hf = 0; hf < D / 64; ++hf)
+            tma_load_2d(kd + hf * KHALF, &k_map, static_cast<int32_t>(e0 % a.k_tok) + hf * 64,
+                        static_cast<int32_t>(e0 / a.k_tok), &full_bar[slot]);
+        }
+      } else {
+        for (int r = lane; r < nr; r += 32)
+          bulk_copy_g2s(kd + r * KSTR, a.k + kb + static_cast<int64_t>(rs + r) * a.k_tok, VSTR, &full_bar[slot]);
+      }
+      if (a.v_tma) {
+        if (lane == 0) {
+          const int64_t e0 = vb + static_cast<int64_t>(rs) * a.v_tok;   // first element of the stage
+          tma_load_2d(vd, &v_map, static_cast<int32_t>(e0 % a.v_tok), static_cast<int32_t>(e0 / a.v_tok),
+                      &full_bar[slot]);
+        }
+      } else if (vc) {
         if (lane == 0) bulk_copy_g2s(vd, a.v + vb + static_cast<int64_t>(rs) * a.v_tok, nr * VSTR, &full_bar[slot]);
       } else {
         for (int r = lane; r < nr; r += 32)
@@ -232,15 +270,29 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const Decod
       ia_cur = ia_next;
       ib_cur = ib_next;
       const int tr0 = r0 + st * kStageRows + warp * kTileRows;   // first row of this warp's tile
-      const uint8_t* kt = ks + slot * kStageRows * KSTR + warp * kTileRows * KSTR;
+      const uint8_t* kt = ks + slot * kStageRows * KSTR + warp * kTileRows * (KT ? 128 : KSTR);
       const uint8_t* vt = vs + slot * kStageRows * VSTR + warp * kTileRows * VSTR;
       if (tr0 < r1) {                                            // (uniform)
         float c[4] = {0.f, 0.f, 0.f, 0.f};
-        const uint8_t* ka = kt + g * KSTR + 4 * t;
+        if constexpr (KT) {
+          // row g (and g + 8) of the warp's 16, swizzled: chunk c of a
+          // 128-byte row sits at chunk c ^ (row mod 8) = c ^ g
+          const uint8_t* kr = kt + g * 128 + 4 * t;
 #pragma unroll
-        for (int k = 0; k < KS; ++k)
-          mma16816(c, lds32(ka + 32 * k), lds32(ka + 8 * KSTR + 32 * k), lds32(ka + 32 * k + 16),
-                   lds32(ka + 8 * KSTR + 32 * k + 16), qb[k][0], qb[k][1]);
+          for (int k = 0; k < KS; ++k) {
+            const uint8_t* kh = kr + (k >> 2) * KHALF;
+            const int c0 = 2 * (k & 3);
+            const int o0 = ((c0 ^ g) << 4), o1 = (((c0 + 1) ^ g) << 4);
+            mma16816(c, lds32(kh + o0), lds32(kh + 8 * 128 + o0), lds32(kh + o1), lds32(kh + 8 * 128 + o1),
+                     qb[k][0], qb[k][1]);
+          }
+        } else {
+          const uint8_t* ka = kt + g * KSTR + 4 * t;
+#pragma unroll
+          for (int k = 0; k < KS; ++k)
+            mma16816(c, lds32(ka + 32 * k), lds32(ka + 8 * KSTR + 32 * k), lds32(ka + 32 * k + 16),
+                     lds32(ka + 8 * KSTR + 32 * k + 16), qb[k][0], qb[k][1]);
+        }
         // rows g and g + 8: inside the split, and a kept slot
         const int ra = tr0 + g, rb = tr0 + g + 8;
         const bool oka = ra < r1 && (idx == nullptr || ia >= 0);
@@ -434,25 +486,26 @@ cudaError_t launch_selftest_wait(uint64_t limit_ns, int32_t* status, cudaStream_
   return cudaGetLastError();
 }
 
-template <int DPL>
-cudaError_t launch_decode_d(const DecodeArgs& a, cudaStream_t stream) {
+template <int DPL, bool KT>
+cudaError_t launch_decode_dk(const DecodeArgs& a, const CUtensorMap& kmap, const CUtensorMap& vmap,
+                             cudaStream_t stream) {
   const int64_t grid1 = static_cast<int64_t>(a.n_units) * a.n_splits;
   const int64_t warps2 = static_cast<int64_t>(a.n_units) * a.G;
   const unsigned grid2 = static_cast<unsigned>((warps2 * 32 + 255) / 256);
-  const int smem = decode_smem_bytes(a.d);
+  const int smem = KT ? decode_smem_bytes_kt(a.d) : decode_smem_bytes(a.d);
   cudaError_t e;
   if (grid1 == 0) {                                  // no rows anywhere: the merge writes zeros
     decode_combine_kernel<DPL><<<grid2, 256, 0, stream>>>(a);
     return cudaGetLastError();
   }
   if (a.G <= 4) {
-    e = cudaFuncSetAttribute(decode_partial_kernel<DPL, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    e = cudaFuncSetAttribute(decode_partial_kernel<DPL, 4, KT>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    decode_partial_kernel<DPL, 4><<<static_cast<unsigned>(grid1), kDecThreads, smem, stream>>>(a);
+    decode_partial_kernel<DPL, 4, KT><<<static_cast<unsigned>(grid1), kDecThreads, smem, stream>>>(a, kmap, vmap);
   } else {
-    e = cudaFuncSetAttribute(decode_partial_kernel<DPL, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    e = cudaFuncSetAttribute(decode_partial_kernel<DPL, 8, KT>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    decode_partial_kernel<DPL, 8><<<static_cast<unsigned>(grid1), kDecThreads, smem, stream>>>(a);
+    decode_partial_kernel<DPL, 8, KT><<<static_cast<unsigned>(grid1), kDecThreads, smem, stream>>>(a, kmap, vmap);
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
@@ -460,9 +513,14 @@ cudaError_t launch_decode_d(const DecodeArgs& a, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream) {
+cudaError_t launch_decode(const DecodeArgs& a, const CUtensorMap& kmap, const CUtensorMap& vmap,
+                          cudaStream_t stream) {
   if (a.n_units == 0) return cudaSuccess;
-  return a.d == 128 ? launch_decode_d<4>(a, stream) : launch_decode_d<2>(a, stream);
+  if (a.k_tma)
+    return a.d == 128 ? launch_decode_dk<4, true>(a, kmap, vmap, stream)
+                      : launch_decode_dk<2, true>(a, kmap, vmap, stream);
+  return a.d == 128 ? launch_decode_dk<4, false>(a, kmap, vmap, stream)
+                    : launch_decode_dk<2, false>(a, kmap, vmap, stream);
 }
 
 }  // namespace rolekv

@@ -152,9 +152,16 @@ struct DecodeArgs {
   int32_t* status;
   // element extents (checked build)
   int64_t ext_q, ext_k, ext_v, ext_keep, ext_part, ext_out;
+  int32_t k_tma;                    // K stages through the tensor map (swizzled halves)
+  int32_t v_tma;                    // V stages through the tensor map (strided rows)
 };
 
-cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
+// kmap: a tensor map over K's token rows (box: 64 rows x 64 columns, 128-byte
+// swizzle), used when a.k_tma is set; vmap: one over V's token rows (box: 64
+// rows x d, no swizzle), used when a.v_tma is set (V rows strided, as in a
+// packed varlen cache).
+cudaError_t launch_decode(const DecodeArgs& a, const CUtensorMap& kmap, const CUtensorMap& vmap,
+                          cudaStream_t stream);
 cudaError_t launch_selftest_wait(uint64_t limit_ns, int32_t* status, cudaStream_t stream);
 
 // Compaction -----------------------------------------------------------------

@@ -180,6 +180,24 @@ int make_row_map(CUtensorMap* map, const rolekv_tensor& t, int64_t span, int box
   return ROLEKV_OK;
 }
 
+// A map over V's token rows for the decode producer (box: 64 rows x d, no
+// swizzle: the consumers read V rows packed), used when the rows are strided.
+// Returns false when the layout does not suit a tensor map (the producer then
+// copies row by row).
+bool make_decode_v_map(CUtensorMap* map, const rolekv_tensor& v, int64_t span, int d) {
+  auto fn = encode_fn();
+  if (fn == nullptr || v.s_tok == d || v.s_layer % v.s_tok != 0 || v.s_seq % v.s_tok != 0) return false;
+  const int64_t rows = (span + v.s_tok - 1) / v.s_tok;
+  if (rows >= (int64_t(1) << 31)) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(v.s_tok), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(v.s_tok) * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(d), 64};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(v.ptr), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 int num_sms() {
   static int sms = 0;
   if (sms == 0) {
@@ -863,9 +881,22 @@ int decode_attention(const rolekv_batch* batch, rolekv_tensor q, rolekv_tensor k
     a.ext_part = static_cast<int64_t>(workspace_bytes / sizeof(float));
     a.ext_out = static_cast<int64_t>(bi.L) * bi.b * bi.Hq * bi.d;
   }
+  CUtensorMap kmap, vmap;
+  std::memset(&kmap, 0, sizeof(kmap));
+  std::memset(&vmap, 0, sizeof(vmap));
+  if (total > 0) {
+    const int64_t rows = bi.varlen ? total : m_max;
+    a.v_tma = make_decode_v_map(&vmap, v_cache, tensor_span(v_cache, bi.L, bi.b, bi.Hkv, rows, bi.d, bi.varlen),
+                                bi.d) ? 1 : 0;
+    // K through a tensor map when its layout suits one (else row by row)
+    const bool k_ok = k_cache.s_layer % k_cache.s_tok == 0 && (bi.varlen || k_cache.s_seq % k_cache.s_tok == 0);
+    if (k_ok && make_row_map(&kmap, k_cache, tensor_span(k_cache, bi.L, bi.b, bi.Hkv, rows, bi.d, bi.varlen), 64) ==
+                    ROLEKV_OK)
+      a.k_tma = 1;                                 // (on failure, row-by-row copies)
+  }
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   stage_begin();
-  cudaError_t e = launch_decode(a, st);
+  cudaError_t e = launch_decode(a, kmap, vmap, st);
   if (e != cudaSuccess) return cuda_fail(e, "decode_attention");
   stage_mark(st);
   return ROLEKV_OK;

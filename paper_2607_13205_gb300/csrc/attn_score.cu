@@ -346,6 +346,35 @@ __device__ __forceinline__ void rowstats_tile(const uint32_t* r, int t0, int pos
   }
 }
 
+// One NCOL-key slice of pass 1 for the row at `pos` (keys t0 .. t0+NCOL-1,
+// raw logits r, overwritten at the causal edge); (m2, l) as in
+// rowstats_tile.  Keys past the row's own position become -inf, so every
+// slice takes the same path: one packed sum against the current reference,
+// redone against the slice's maximum when there is no reference yet (the
+// chunk's first slice) or the sum shows a much larger logit.
+template <int NCOL>
+__device__ __forceinline__ void rowstats_slice(uint32_t* r, int t0, int pos, float c1,
+                                               float& m2, float& l) {
+  if (pos < 0 || t0 > pos) return;
+  if (t0 + NCOL - 1 > pos) {
+    const int last = pos - t0;
+#pragma unroll
+    for (int i = 0; i < NCOL; ++i)
+      if (i > last) r[i] = 0xFF800000u;          // -inf
+  }
+  if (m2 > -INFINITY) {
+    const float s = sum_exp2_shift<NCOL>(r, c1, m2);
+    if (s <= 1.0e18f) {
+      l += s;
+      return;
+    }
+  }
+  const float mnew = fmaxf(m2, max_cols<NCOL>(r) * c1);
+  const float s = sum_exp2_shift<NCOL>(r, c1, mnew);
+  l = l * fast_exp2(m2 - mnew) + s;
+  m2 = mnew;
+}
+
 // Pass 1 epilogue: the thread owns one query row and NCOL keys of every tile.
 // With two row tiles, two parts share each tile (NCOL = 64 keys each); with
 // one, all four parts share it (NCOL = 32).  The parts merge at the end.
@@ -869,33 +898,41 @@ __device__ __forceinline__ FItem fused_item(const ScoreArgs& a, int item) {
   return it;
 }
 
+// Descriptor `d` moved `bytes` further into shared memory.  The start-address
+// field is the low 14 bits (16-byte units) and every operand stays inside
+// shared memory, so the add never carries out of the low word.
+__device__ __forceinline__ uint64_t desc_plus(uint64_t d, uint32_t bytes) {
+  const uint32_t lo = static_cast<uint32_t>(d) + (bytes >> 4);
+  return (d & 0xFFFFFFFF00000000ull) | lo;
+}
+
 template <int D>
-__device__ __forceinline__ void issue_mma_rows_on_lanes(uint32_t qbase, uint32_t kbase,
+__device__ __forceinline__ void issue_mma_rows_on_lanes(uint64_t dq, uint64_t dk,
                                                         uint32_t dcol, int nrt) {
   using C = FCfg<D>;
   const uint32_t idesc = idesc_bf16_f32(128, kTileKeys);
   for (int rt = 0; rt < nrt; ++rt) {
+    const uint64_t dqr = desc_plus(dq, rt * 128 * 128);
 #pragma unroll
     for (int ks = 0; ks < C::kKSteps; ++ks) {
       const uint32_t koff = (ks & 3) * 32;
-      const uint64_t ad =
-          sdesc_kmajor_sw128(qbase + (ks >> 2) * C::kQHalfBytes + rt * 128 * 128 + koff);
-      const uint64_t bd = sdesc_kmajor_sw128(kbase + (ks >> 2) * C::kKHalfBytes + koff);
+      const uint64_t ad = desc_plus(dqr, (ks >> 2) * C::kQHalfBytes + koff);
+      const uint64_t bd = desc_plus(dk, (ks >> 2) * C::kKHalfBytes + koff);
       mma_bf16_ss(dcol + rt * kTileKeys, ad, bd, idesc, ks > 0 ? 1u : 0u);
     }
   }
 }
 
 template <int D>
-__device__ __forceinline__ void issue_mma_keys_on_lanes(uint32_t qbase, uint32_t kbase,
+__device__ __forceinline__ void issue_mma_keys_on_lanes(uint64_t dq, uint64_t dk,
                                                         uint32_t dcol, int nrows_pad) {
   using C = FCfg<D>;
   const uint32_t idesc = idesc_bf16_f32(128, nrows_pad);
 #pragma unroll
   for (int ks = 0; ks < C::kKSteps; ++ks) {
     const uint32_t koff = (ks & 3) * 32;
-    const uint64_t ad = sdesc_kmajor_sw128(kbase + (ks >> 2) * C::kKHalfBytes + koff);
-    const uint64_t bd = sdesc_kmajor_sw128(qbase + (ks >> 2) * C::kQHalfBytes + koff);
+    const uint64_t ad = desc_plus(dk, (ks >> 2) * C::kKHalfBytes + koff);
+    const uint64_t bd = desc_plus(dq, (ks >> 2) * C::kQHalfBytes + koff);
     mma_bf16_ss(dcol, ad, bd, idesc, ks > 0 ? 1u : 0u);
   }
 }
@@ -1039,7 +1076,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (!mbar_wait(sh.q_full, quse & 1, sh.abort_flag, a.status)) break;
         ++quse;
-        const uint32_t qbase = smem_u32(sh.q);
+        const uint64_t dq = sdesc_kmajor_sw128(smem_u32(sh.q));
         bool nl_ready = false;
         for (int pass = fa.single; pass < 2 && ok; ++pass)
           for (int kt = kt0; kt < kt1; ++kt) {
@@ -1051,11 +1088,11 @@ __global__ void __launch_bounds__(kThreads, 1)
               break;
             }
             tc_fence_after();
-            const uint32_t kbase = smem_u32(sh.k + kslot * C::kKTileBytes);
+            const uint64_t dk = sdesc_kmajor_sw128(smem_u32(sh.k + kslot * C::kKTileBytes));
             if (pass == 0) {
-              issue_mma_rows_on_lanes<D>(qbase, kbase, tmem + ab * 256, nrt);
+              issue_mma_rows_on_lanes<D>(dq, dk, tmem + ab * 256, nrt);
             } else {
-              issue_mma_keys_on_lanes<D>(qbase, kbase, tmem + ab * 256, p2n);
+              issue_mma_keys_on_lanes<D>(dq, dk, tmem + ab * 256, p2n);
               // add the rows' normalisers (once the epilogue has written them)
               if (!nl_ready) {
                 if (!mbar_wait(sh.lse_ready, lpop & 1, sh.abort_flag, a.status)) {
@@ -1129,14 +1166,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         ok = __all_sync(0xffffffffu, mbar_wait(&sh.acc_full[ab], (pair >> 1) & 1, sh.abort_flag, a.status));
         if (!ok) break;
         tc_fence_after();
-        uint32_t r[32];
-        for (int h = 0; h < p1cols / 32; ++h) {
-          tmem_load_cols<32>(tmem + lane_base + ab * 256 + col1 + h * 32, r);
-          if (h + 1 == p1cols / 32) {
+        uint32_t r[64];
+        for (int h = 0; h < p1cols / 64; ++h) {
+          tmem_load_cols<64>(tmem + lane_base + ab * 256 + col1 + h * 64, r);
+          if (h + 1 == p1cols / 64) {
             tc_fence_before();
             mbar_arrive(&sh.acc_empty[ab]);
           }
-          rowstats_tile<32>(r, kt * kTileKeys + key1 + h * 32, pos, c1, m2, l);
+          rowstats_slice<64>(r, kt * kTileKeys + key1 + h * 64, pos, c1, m2, l);
         }
       }
       if (!ok) break;

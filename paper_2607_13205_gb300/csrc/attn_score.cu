@@ -349,9 +349,8 @@ __device__ __forceinline__ void rowstats_tile(const uint32_t* r, int t0, int pos
 // One NCOL-key slice of pass 1 for the row at `pos` (keys t0 .. t0+NCOL-1,
 // raw logits r, overwritten at the causal edge); (m2, l) as in
 // rowstats_tile.  Keys past the row's own position become -inf, so every
-// slice takes the same path: one packed sum against the current reference,
-// redone against the slice's maximum when there is no reference yet (the
-// chunk's first slice) or the sum shows a much larger logit.
+// slice takes the same branch-free path: the reference moves to the slice's
+// maximum first (three-input max on the ALU), then one packed sum against it.
 template <int NCOL>
 __device__ __forceinline__ void rowstats_slice(uint32_t* r, int t0, int pos, float c1,
                                                float& m2, float& l) {
@@ -361,13 +360,6 @@ __device__ __forceinline__ void rowstats_slice(uint32_t* r, int t0, int pos, flo
 #pragma unroll
     for (int i = 0; i < NCOL; ++i)
       if (i > last) r[i] = 0xFF800000u;          // -inf
-  }
-  if (m2 > -INFINITY) {
-    const float s = sum_exp2_shift<NCOL>(r, c1, m2);
-    if (s <= 1.0e18f) {
-      l += s;
-      return;
-    }
   }
   const float mnew = fmaxf(m2, max_cols<NCOL>(r) * c1);
   const float s = sum_exp2_shift<NCOL>(r, c1, mnew);

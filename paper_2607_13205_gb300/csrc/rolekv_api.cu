@@ -10,7 +10,7 @@
 #include <cstdint>
 #include <cstdio>
 #include <cstring>
-#include <mutex>
+#include <mutex>  // std::call_once
 
 #include <nvtx3/nvToolsExt.h>
 
@@ -513,26 +513,15 @@ static __device__ __align__(256) unsigned char rolekv_noalloc_scratch[kNoAllocSc
 namespace rolekv {
 namespace {
 
-constexpr int kMaxDevices = 64;
-std::mutex g_scratch_mutex;
-void* g_scratch_ptr[kMaxDevices] = {};
-
-// Device address of the scratch array on the current device.  The host-side
-// name of the array is only a stand-in, so the address is looked up once per
-// device, with that device current, and cached.
+// Device address of the scratch array in the current context.  The host-side
+// name of the array is only a stand-in; the address is looked up on every
+// call (a cheap runtime query), so a context that was reset and made again
+// never sees an address from the old one.
 int noalloc_scratch(void** out) {
-  int dev = -1;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
-  if (dev < 0 || dev >= kMaxDevices) return fail(ROLEKV_ERR_UNSUPPORTED, "device %d out of range", dev);
-  std::lock_guard<std::mutex> lock(g_scratch_mutex);
-  if (g_scratch_ptr[dev] == nullptr) {
-    void* ptr = nullptr;
-    e = cudaGetSymbolAddress(&ptr, rolekv_noalloc_scratch);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(scratch)");
-    g_scratch_ptr[dev] = ptr;
-  }
-  *out = g_scratch_ptr[dev];
+  void* ptr = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&ptr, rolekv_noalloc_scratch);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(scratch)");
+  *out = ptr;
   return ROLEKV_OK;
 }
 

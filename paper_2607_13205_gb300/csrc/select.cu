@@ -121,6 +121,9 @@ struct SelShared {
   uint32_t partial_ties;   // buckets with more threshold ties than slots left
   int32_t slack;           // SLACK policy: slots left to fill by score
   uint32_t elig_mask;      // roles taking part in the split (bit r)
+  int32_t sfast;           // SLACK: the fill's first digit is known (below)
+  uint32_t sprefix;        // SLACK: shared top bit and first digit of the fill threshold
+  int32_t sneed;           // SLACK: tokens at that digit still to fill
 };
 
 // Slots 4g .. 4g+3 of a score row; slots outside [off, off + n) read -inf.
@@ -480,6 +483,101 @@ __device__ void descend_first(const SelectArgs& a, SelShared& S, const uint32_t*
   }
 }
 
+// SLACK policy: the first digit of the fill threshold, from the same pass-1
+// histograms, once every bucket's first digit is known.  The tokens the fill
+// ranks are the eligible ones no bucket keeps; per first-digit bin they are
+// a role's whole bin (its bucket keeps nothing, or the bin lies below the
+// bucket's digit), none (the bucket keeps the bin), or the bin less the
+// need[b] tokens the bucket keeps at its own digit.  Every thread counts a
+// few bins into `cnt` (shared memory, 2^NB ints); then warp 0 locates the
+// bin holding the slack-th token from the top: each lane sums a contiguous
+// range, the lanes' totals from the top locate the range, and the warp
+// splits that range.  On success sprefix / sneed are set and sfast = 1;
+// otherwise the fill takes its full-pass rounds.  Every thread calls it.
+template <int NB, int NT>
+__device__ void slack_first(const SelectArgs& a, SelShared& S, const uint32_t* hist16, int* cnt,
+                            int list_cap) {
+  constexpr int nbins = 1 << NB;
+  constexpr int bpl = nbins / 32;        // bins per lane
+  constexpr int wpr = 1 << (NB - 1);     // histogram words (two bins each) per role
+  constexpr int sh0 = 31 - NB;
+  const int tid = threadIdx.x, lane = tid & 31;
+  for (int x = tid; x < nbins; x += NT) {
+    int c = 0;
+    for (int r = 0; r < a.n_roles; ++r) {
+      if (!((S.elig_mask >> r) & 1u)) continue;
+      const uint32_t code = static_cast<uint32_t>(S.code_of_role[r]);
+      if (code == kCodeKeep) continue;
+      const uint32_t w = hist16[r * wpr + (x >> 1)];
+      const int h = static_cast<int>((x & 1) ? (w >> 16) : (w & 0xFFFFu));
+      if (code >= static_cast<uint32_t>(kR)) {
+        c += h;                                  // its bucket keeps nothing
+      } else {
+        const int D = static_cast<int>((S.prefix[code] >> sh0) & (nbins - 1));
+        c += x < D ? h : (x == D ? h - S.need[code] : 0);
+      }
+    }
+    cnt[x] = c;
+  }
+  __syncthreads();
+  if (tid < 32) {
+    const int need = S.slack;
+    int mine = 0;
+#pragma unroll 8
+    for (int i = 0; i < bpl; ++i) mine += cnt[lane * bpl + ((i + lane) & (bpl - 1))];
+    int incl = mine;                             // tokens in this lane's bins or above
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_down_sync(0xffffffffu, incl, o);
+      if (lane + o < 32) incl += v;
+    }
+    const int above = incl - mine;
+    const unsigned who = __ballot_sync(0xffffffffu, above < need && above + mine >= need);
+    if (who != 0) {
+      const int F = __ffs(who) - 1;
+      const int aboveF = __shfl_sync(0xffffffffu, above, F);
+      const int needF = need - aboveF;
+      // the winning range split over the warp: bpl / 32 bins a lane
+      constexpr int per = bpl / 32 > 0 ? bpl / 32 : 1;
+      int c2[per];
+      int part = 0;
+#pragma unroll
+      for (int i = 0; i < per; ++i) {
+        c2[i] = (lane * per + i < bpl) ? cnt[F * bpl + lane * per + i] : 0;
+        part += c2[i];
+      }
+      int incl2 = part;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int v = __shfl_down_sync(0xffffffffu, incl2, o);
+        if (lane + o < 32) incl2 += v;
+      }
+      const int above2 = incl2 - part;
+      const unsigned who2 = __ballot_sync(0xffffffffu, above2 < needF && above2 + part >= needF);
+      if (who2 != 0 && lane == __ffs(who2) - 1) {
+        int acc = above2, fd = -1, nd = 0, at = 0;
+#pragma unroll
+        for (int i = per - 1; i >= 0; --i) {
+          if (fd < 0 && acc + c2[i] >= needF) {
+            fd = F * bpl + lane * per + i;
+            nd = needF - acc;
+            at = c2[i];
+          }
+          acc += c2[i];
+        }
+        if (fd >= 0 && at <= list_cap) {
+          S.sprefix = (S.top_and & 0x80000000u) | (static_cast<uint32_t>(fd) << sh0);
+          S.sneed = nd;
+          S.sfast = 1;
+        }
+      }
+    }
+  }
+  __syncthreads();
+  for (int x = tid; x < nbins; x += NT) cnt[x] = 0;
+  __syncthreads();
+}
+
 // descend_first for the streaming mode's 32-bit bins: lane L owns bins
 // L * 2^NB / 32 ..; the lanes' totals locate the lane holding the threshold,
 // then the warp splits that lane's bins (at most 64, two per lane).
@@ -664,6 +762,7 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
     S.top_or = 0u;
     S.slack = 0;
     S.elig_mask = 0u;
+    S.sfast = 0;
   }
   for (int x = tid; x < kR * 256; x += NT) (&S.hist[0][0])[x] = 0;
   {
@@ -807,6 +906,16 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
         descend_first<10>(a, S, hist16, warp, lane);
     }
     __syncthreads();
+  }
+  // SLACK: the fill's first digit from the same histograms, before their
+  // region becomes the candidate list (in-memory rows; 16-bit bins)
+  if (!STREAM && S.slack > 0 && !S.general) {
+    // (S.hist, zero until the refinement rounds, serves as the bin counts)
+    static_assert(kR * 256 >= 2048, "bin counts for an 11-bit digit");
+    if (nb == 11)
+      slack_first<11, NT>(a, S, hist16, &S.hist[0][0], list_cap);
+    else
+      slack_first<10, NT>(a, S, hist16, &S.hist[0][0], list_cap);
   }
   // While the keys at the buckets' first digits overflow the list (scores in
   // a narrow range, such as page bounds), one full pass per 8 more bits.
@@ -1065,10 +1174,137 @@ __global__ void __launch_bounds__(NT, 1024 / NT) select_kernel(const SelectArgs 
   }
 
   // ---- SLACK: the slots saturated buckets left go to the best-scoring
-  // tokens of eligible roles not kept yet (ties to the lower index): four
-  // 8-bit rounds over all slots for the slack-th largest such key, in the
-  // state of bucket 0, whose own selection is complete.
-  if (S.slack > 0) {
+  // tokens of eligible roles not kept yet (ties to the lower index).  With
+  // the fill's first digit known (sfast), one pass keeps such tokens above
+  // it and lists those at it; the remaining bits are resolved over the list
+  // in the state of bucket 0, whose own selection is complete.
+  if (!STREAM && S.slack > 0 && S.sfast) {
+    const uint32_t elig = S.elig_mask;
+    const int sh0 = 31 - nb;
+    const uint32_t bmask = (1u << nb) - 1u;
+    const uint32_t DS = (S.sprefix >> sh0) & bmask;
+    if (tid == 0) {
+      S.list_n = 0;
+      S.tie_n = 0;
+      S.partial_ties = 0;
+      S.prefix[0] = S.sprefix;
+      S.need[0] = S.sneed;
+      S.thr[0] = 0xFFFFFFFFu;
+    }
+    for (int x = tid; x < 256; x += NT) S.hist[0][x] = 0;
+    __syncthreads();
+    for (int i = 0; i < iters; ++i) {
+      const int g = i * NT + tid;
+      uint32_t m4 = 0, c4 = 0;
+      if (g < ngroups) {
+        const uint4 kv = keys4[g];
+        const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
+        const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
+        const uint32_t fb = floor_bits(4 * g - off, v.nf, n);
+        const uint32_t kb = (bits[g >> 3] >> (4 * (g & 7))) & 0xFu;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t r = (rw >> (8 * j)) & 0xFFu;
+          if (r >= static_cast<uint32_t>(kR) || !((elig >> r) & 1u) || ((fb | kb) >> j) & 1u) continue;
+          const uint32_t d = (kk[j] >> sh0) & bmask;
+          m4 |= static_cast<uint32_t>(d > DS) << j;
+          c4 |= static_cast<uint32_t>(d == DS) << j;
+        }
+        if (m4) atomicOr(&bits[g >> 3], m4 << (4 * (g & 7)));
+      }
+      const int nc = __popc(c4);
+      const unsigned b1 = __ballot_sync(0xffffffffu, nc >= 1);
+      if (b1 != 0) {
+        const unsigned b2 = __ballot_sync(0xffffffffu, nc >= 2);
+        const unsigned b3 = __ballot_sync(0xffffffffu, nc >= 3);
+        const unsigned b4 = __ballot_sync(0xffffffffu, nc >= 4);
+        const unsigned lt = (1u << lane) - 1u;
+        int base = 0;
+        if (lane == 0) base = atomicAdd(&S.list_n, __popc(b1) + __popc(b2) + __popc(b3) + __popc(b4));
+        base = __shfl_sync(0xffffffffu, base, 0);
+        int pos = base + __popc(b1 & lt) + __popc(b2 & lt) + __popc(b3 & lt) + __popc(b4 & lt);
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          if ((c4 >> j) & 1u) {
+            if (pos < list_cap) list[pos] = static_cast<uint32_t>(4 * g + j);
+            ++pos;
+          }
+      }
+    }
+    __syncthreads();
+    // (the histograms bound the listed count by list_cap)
+    const int m = S.list_n < list_cap ? S.list_n : list_cap;
+    for (int lo = sh0; lo > 0;) {
+      const int d = lo < 8 ? lo : 8;
+      const int shift = lo - d;
+      for (int e = tid; e < m; e += NT) {
+        const uint32_t key = keys[list[e]];
+        if ((key >> lo) == (S.prefix[0] >> lo)) atomicAdd(&S.hist[0][(key >> shift) & ((1u << d) - 1u)], 1);
+      }
+      __syncthreads();
+      if (warp == 0) descend(S, 0, lane, shift);
+      __syncthreads();
+      lo = shift;
+    }
+    const uint32_t T = S.thr[0], P = S.prefix[0];
+    const int need = S.need[0];
+    const bool partial = S.partial_ties & 1u;
+    for (int e = tid; e < m; e += NT) {
+      const uint32_t slot = list[e];
+      const uint32_t key = keys[slot];
+      if (key >= T) {
+        atomicOr(&bits[slot >> 5], 1u << (slot & 31u));
+      } else if (partial && key == P) {
+        const int t = atomicAdd(&S.tie_n, 1);
+        if (t < kTieCap) S.ties[t] = slot;
+      }
+    }
+    __syncthreads();
+    const int nt = S.tie_n;
+    if (partial && nt <= kTieCap) {
+      // index-order rank among the fill's ties
+      for (int t = tid; t < nt; t += NT) {
+        const uint32_t slot = S.ties[t];
+        int rank = 0;
+        for (int x = 0; x < nt; ++x) rank += S.ties[x] < slot;
+        if (rank < need) atomicOr(&bits[slot >> 5], 1u << (slot & 31u));
+      }
+      __syncthreads();
+    } else if (partial) {
+      // more ties than the shared list holds: rank them over all slots
+      auto tie_mask = [&](int q) {
+        uint32_t mk = 0;
+#pragma unroll
+        for (int gg = 0; gg < 8; ++gg) {
+          const int g = 8 * q + gg;
+          if (g >= ngroups) break;
+          const uint4 kv = keys4[g];
+          const uint32_t kk[4] = {kv.x, kv.y, kv.z, kv.w};
+          const uint32_t rw = load_roles(v.rp, off, n, g, v.rvec);
+          const uint32_t fb = floor_bits(4 * g - off, v.nf, n);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const uint32_t r = (rw >> (8 * j)) & 0xFFu;
+            const int slot = 4 * g + j;
+            if (kk[j] == P && r < static_cast<uint32_t>(kR) && ((elig >> r) & 1u) && !((fb >> j) & 1u) &&
+                !((bits[slot >> 5] >> (slot & 31)) & 1u))
+              mk |= 1u << (4 * gg + j);
+          }
+        }
+        return mk;
+      };
+      scan_words<NT>(nwords, tie_mask, [&](int q, uint32_t mk, int rank) {
+        uint32_t keepm = 0;
+        while (mk != 0 && rank < need) {
+          const uint32_t low = mk & (0u - mk);
+          keepm |= low;
+          mk ^= low;
+          ++rank;
+        }
+        if (keepm) bits[q] |= keepm;
+      }, S.warp_tot);
+    }
+  } else if (S.slack > 0) {
     const uint32_t elig = S.elig_mask;
     auto candidate = [&](uint32_t rw, uint32_t fb, int g, int j) {
       const uint32_t r = (rw >> (8 * j)) & 0xFFu;

@@ -460,13 +460,17 @@ def test_role_alloc_select_bit_exact(case):
 
 
 NARROW_CASES = [
-    # (name, n, policy, pool_k, spread): page-constant scores in [2, 2 + spread)
+    # (name, n, policy, pool_k, spread[, budget]): page-constant scores in [2, 2 + spread)
     ("narrow_quota", 20000, 0, 1, 0.2),
     ("narrow_global_stream", 70000, 1, 3, 0.2),
     ("narrow_global_pool7", 20000, 1, 7, 0.2),
     ("narrow_fair_short", 9000, 2, 1, 0.2),
     ("constant_global", 20000, 1, 1, 0.0),
     ("constant_quota_pool5", 12000, 0, 5, 0.0),
+    # SLACK fill: its first digit holds a few thousand page-tied keys (listed,
+    # then ranked), or every key (the list overflows: full-pass rounds)
+    ("narrow_slack_b50", 20000, 3, 1, 2.0, 0.5),
+    ("constant_slack_pool3_b50", 16000, 3, 3, 0.0, 0.5),
 ]
 
 
@@ -476,7 +480,8 @@ def test_select_narrow_page_constant_scores(case):
     Quest page bounds are): most keys share the first digit, so the selector
     takes extra digit rounds before listing candidates; a constant row leaves
     only ties.  Bit-exact against the oracle on the same scores."""
-    name, n, policy, pool_k, spread = case
+    name, n, policy, pool_k, spread = case[:5]
+    B = case[5] if len(case) > 5 else 0.10
     w = _w("llama8b", L=1, b=2, Hq=8, Hkv=2, n=n)
     roles_np = I.workload_roles(w, 3)
     batch = lib_batch(w, DEV)
@@ -485,7 +490,6 @@ def test_select_narrow_page_constant_scores(case):
     pages = 2.0 + spread * torch.rand((batch.n_units, npages), generator=g)
     sc = pages.repeat_interleave(16, dim=1)[:, :n].reshape(batch.score_shape()).contiguous()
     scores = sc.to(DEV)
-    B = 0.10
     params = R.select_params(B, I.PAPER_ALPHA, alpha_key=0.0, key_role=I.ROLE_KEY, policy=policy)
     keep = torch.full(batch.kept_shape(B), -7, dtype=torch.int32, device=DEV)
     per_role = torch.full((batch.n_units, I.N_ROLES), -1, dtype=torch.int32, device=DEV)

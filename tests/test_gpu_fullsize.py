@@ -155,6 +155,45 @@ def _check_ceil_select(w, B, r, units):
         assert list(pr[u]) == per
 
 
+def _check_slack_select(w, B, r, units, alpha_key=0.02):
+    """The SLACK fill (first-round quotas, the slack of saturated buckets to
+    the best-scoring unkept tokens of eligible roles) on the kernel's own
+    scores: every unit keeps exactly min(ceil(B n), eligible) tokens in an
+    ascending row counted per role; bit-exact against the oracle on the
+    sampled units."""
+    batch = lib_batch(w, DEV)
+    ob = oracle_batch(w)
+    pre = torch.as_tensor(r["scores"], device=DEV)
+    params = R.select_params(B, I.PAPER_ALPHA, alpha_key, I.ROLE_KEY, policy=R.POLICY_SLACK)
+    keep = torch.full(batch.kept_shape(B), -7, dtype=torch.int32, device=DEV)
+    per_role = torch.empty((batch.n_units, I.N_ROLES), dtype=torch.int32, device=DEV)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    R.role_alloc_select(batch, pre, torch.as_tensor(r["roles"], device=DEV), params, keep,
+                        pool_k=w.pool_k, kept_per_role=per_role, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    keep_np, pr = keep.cpu().numpy(), per_role.cpu().numpy()
+    kept_off = ob.kept_offsets(B)
+    alpha = list(I.PAPER_ALPHA)
+    alpha[I.ROLE_KEY] = alpha_key
+    for u in range(ob.n_units):
+        s = ob.unit(u)[1]
+        n = ob.seqlens[s]
+        row = _unit_rows(ob, keep_np, u, kept_off)
+        kept = row[row >= 0]
+        assert np.all(row[kept.size:] == -1) and np.all(np.diff(kept) > 0)
+        counts = np.bincount(np.asarray(ob.roles(r["roles"], s)), minlength=I.N_ROLES)[:I.N_ROLES]
+        eligible = int(sum(c for c, a in zip(counts, alpha) if a > 0))
+        assert kept.size == min(O.kept_count(n, B), eligible), (u, kept.size)
+        assert int(pr[u].sum()) == kept.size
+    for u in units:
+        sc = O.maxpool1d(ob.score_view(r["scores"], u).astype(np.float64), w.pool_k)
+        idx, per = O.select_batch(ob, {u: sc}, r["roles"], I.N_ROLES, I.PAPER_ALPHA, I.ROLE_KEY,
+                                  alpha_key, B, O.POLICY_SLACK)[u]
+        assert np.array_equal(_unit_rows(ob, keep_np, u, kept_off), idx), f"slack unit {u}"
+        assert list(pr[u]) == per
+
+
 def test_long_context_full_size():
     """L=32, b=4, N=32768, 32/8 heads, d=128, W=64, pool 7, B=0.10 (~17 GB K/V)."""
     w = I.WORKLOADS["long"]
@@ -164,6 +203,7 @@ def test_long_context_full_size():
     _check_all_units(w, B, ob, r, 0.0, lambda n: min(w.W, n) * w.G)
     _check_sampled_snapkv(w, B, ob, [0, 517, ob.n_units - 1], r, 0.0)
     _check_ceil_select(w, B, r, [0, 517, ob.n_units - 1])
+    _check_slack_select(w, B, r, [3, 600, ob.n_units - 1])
     _check_one_call(w, B, ob, r, [5, 700, ob.n_units - 2])
 
 

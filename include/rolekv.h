@@ -216,12 +216,11 @@ int snapkv_score(const rolekv_batch* batch, rolekv_tensor q_win, rolekv_tensor k
  *   ROLEKV_ERR_UNSUPPORTED (about 9 MiB for 32 layers x 4 x 8 KV heads at
  *   32768 tokens); with pool_k > 1, scores_prepool is required, because the
  *   pre-pool scores are an output here, not scratch.
- *   Set-up: the first call on each device looks up the array's device address
- *   (cudaGetSymbolAddress) with that device current and caches it for the
- *   rest of the process; make that first call before any stream capture.
- *   The cached address belongs to the device's primary context (the one the
- *   CUDA runtime uses by default): call this entry point only from that
- *   context, and not after cudaDeviceReset on the device.
+ *   Set-up: every call looks up the array's device address in the current
+ *   context (cudaGetSymbolAddress, a cheap runtime query), so a context that
+ *   was reset and made again gets its own array; the first call on a device
+ *   also loads the library's device code there, so make it before any
+ *   stream capture.
  *   Empty batches (no tokens) return ROLEKV_OK without touching any buffer,
  *   as snapkv_score does.
  *   Sharing: every call on a device uses the same array and leaves its
